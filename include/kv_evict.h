@@ -1,0 +1,149 @@
+/*
+ * kv_evict.h -- C ABI of the GB300 (sm_103a) diversified KV-eviction step.
+ *
+ * The step is the end-of-prefill token eviction of "Beyond Mean Attention:
+ * Diversity-Aware, Layer-Wise Scoring for KV Cache Eviction" (Section 3). For every
+ * (request, layer, KV head) -- a "unit" -- it
+ *   1. scores every prefix token i by the attention A[q][i] it receives from the
+ *      observation window, the last W query positions (Section 3.1, Eq. 1);
+ *   2. reduces those scores over the window rows to the mean mu_i (Eq. 1) and the
+ *      sample standard deviation sigma_i (Eq. 3);
+ *   3. max-pools mu and sigma over the candidate tokens (Section 3.1 keeps the
+ *      baselines' max-pooling), forms the base score s_i = mu_i + lambda1 * sigma_i
+ *      (Eq. 2 without the redundancy term), restricts the candidates to the top
+ *      4B tokens by s (Section 3.2), normalises s by its maximum (Eq. 5) and admits
+ *      B tokens greedily by s~_i + lambda2 * corr(i, S) (Eq. 4, Eq. 5);
+ *   4. gathers the kept key/value rows into a compact cache.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  * Symbols: N_L layers, Hq query heads, Hkv KV heads, G = Hq / Hkv (GQA group),
+ *    d = head_dim, W = window, B = budget, n_req requests with prefix lengths L_r,
+ *    SL = sum_r L_r, Lc_r = L_r - W candidate tokens of request r.
+ *  * The window rows of unit (r, l, h) are the G query heads h*G .. h*G+G-1, each
+ *    with its W window queries: n = G*W rows, row index g*W + w, at token position
+ *    L_r - W + w. Causal masking: that row attends to keys 0 .. L_r - W + w.
+ *  * All tensors are dense, row-major, in device memory, allocated and owned by
+ *    the caller. bf16 tensors are passed as uint16_t bit patterns.
+ *      q_win  [N_L][n_req][Hq][W][d]      bf16  window queries (after RoPE)
+ *      k, v   [N_L][Hkv][SL][d]           bf16  prefix keys/values (after RoPE);
+ *                                               request r occupies tokens
+ *                                               off_r .. off_r + L_r - 1,
+ *                                               off_r = L_0 + ... + L_{r-1}
+ *      mu, sigma  packed per request: request r holds [N_L][Hkv][L_r] fp32 at
+ *                 element offset N_L*Hkv*off_r
+ *      indices    [n_req][N_L][Hkv][B] int32, kept candidate positions in
+ *                 ascending order, -1 after the first min(B, Lc_r) entries
+ *      order      [n_req][N_L][Hkv][B] int32, the same positions in admission
+ *                 order (optional)
+ *      margins    [n_req][N_L][Hkv][B] fp32, per admission the gap between the
+ *                 best and the second-best greedy value (optional)
+ *      k_out, v_out [n_req][N_L][Hkv][B+W][d] bf16: rows 0 .. m-1 are the kept
+ *                 candidates in ascending position (m = min(B, Lc_r)), rows
+ *                 m .. m+W-1 the W window tokens, remaining rows zero.
+ *  * Every pointer must be 16-byte aligned; q_win and k additionally 128-byte.
+ *  * stream is a cudaStream_t passed as void*. Every device call is
+ *    asynchronous on that stream and returns after the launches; device-side
+ *    failures (a bounded wait that ran out) are reported by kv_evict_status.
+ *  * Host validation failures return before any launch and write nothing.
+ *  * A plan is immutable after kv_evict_plan and may be used from several host
+ *    threads; a workspace must not be shared by calls that overlap on the GPU.
+ */
+#ifndef KV_EVICT_H
+#define KV_EVICT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  KVE_OK = 0,
+  KVE_EINVAL = 1,   /* invalid argument or unsupported shape (host check)     */
+  KVE_ECUDA = 2,    /* a CUDA runtime/driver call failed                      */
+  KVE_ETIMEOUT = 3, /* a device-side bounded wait ran out (kv_evict_status)   */
+  KVE_ENOMEM = 4    /* host allocation failed                                 */
+} kve_status;
+
+typedef struct {
+  int32_t num_layers;       /* N_L >= 1                                        */
+  int32_t num_q_heads;      /* Hq, a multiple of num_kv_heads                  */
+  int32_t num_kv_heads;     /* Hkv >= 1                                        */
+  int32_t head_dim;         /* d; this build supports d = 128                  */
+  int32_t window;           /* W >= 1, with G*W <= 128                         */
+  int32_t budget;           /* B >= 1 kept candidates per unit (the window is
+                               kept in addition)                               */
+  int32_t pool_kernel;      /* odd k >= 1; max-pool of mu and sigma, stride 1,
+                               window clipped to [0, Lc); 1 = no pooling       */
+  int32_t candidate_factor; /* greedy pool C = min(factor*B, Lc); Section 3.2
+                               uses 4; 0 = every candidate                     */
+  float norm_eps;           /* positive clamp of max_j s_j in Eq. 5            */
+} kve_config;
+
+typedef struct kve_plan kve_plan;
+
+/* Validate cfg and the host array seq_lens[n_req] (every L_r > W), and build the
+ * host-side schedule. *workspace_bytes receives the size of the device workspace
+ * that kv_evict_score and kv_evict_select need (caller-allocated, 256-byte
+ * aligned). The plan owns host memory only. Section 3 defines the shapes. */
+kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens,
+                         int32_t n_req, kve_plan** plan_out,
+                         size_t* workspace_bytes);
+
+void kv_evict_plan_destroy(kve_plan* plan);
+
+/* Test hook: limit (ns) of every device-side bounded wait of later calls with this
+ * plan (default 2e9), and a fault to inject on the host-chosen unit 0:
+ * fault = 1 makes its row statistics never publish, so its column pass waits
+ * out the limit and kv_evict_status reports KVE_ETIMEOUT. fault = 0 is normal. */
+kve_status kv_evict_plan_set_debug(kve_plan* plan, uint64_t wait_limit_ns,
+                                   int32_t fault);
+
+/* Steps 1-2: window attention (Section 3.1 and Eq. 1 context: softmax of the
+ * scaled window-query/key logits over the whole causal prefix, window keys
+ * included), then per token mu (Eq. 1) and sigma (Eq. 3, divisor n - 1; sigma = 0
+ * when n = 1) for every token 0 .. L_r - 1 of every unit. Reads q_win and k,
+ * writes mu and sigma, uses ws as scratch. */
+kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win,
+                          const uint16_t* k, float* mu, float* sigma, void* ws,
+                          void* stream);
+
+/* Step 3: pooling (Section 3.1), base score (Eq. 2), top factor*B candidate pool
+ * (Section 3.2), normalisation (Eq. 5, denominator clamped to norm_eps), greedy
+ * admission by s~ + lambda2 * corr(i, S) (Eq. 4, Eq. 5) with ties broken towards
+ * the lower token position. lambda1 and lambda2 are HOST arrays [N_L] (the
+ * layer-wise coefficients of Section 3.3). Writes indices; order and margins may
+ * be NULL. Uses ws as scratch. */
+kve_status kv_evict_select(const kve_plan* plan, const float* mu,
+                           const float* sigma, const uint16_t* k,
+                           const float* lambda1, const float* lambda2,
+                           int32_t* indices, int32_t* order, float* margins,
+                           void* ws, void* stream);
+
+/* Step 4: compact cache (Section 1: each layer keeps B entries after prefill;
+ * the window tokens are kept as well). Copies key/value rows bit-exactly. */
+kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k,
+                           const uint16_t* v, const int32_t* indices,
+                           uint16_t* k_out, uint16_t* v_out, void* stream);
+
+/* Synchronise the stream, read the device error word of ws and clear it.
+ * Returns KVE_OK, KVE_ETIMEOUT or KVE_ECUDA. */
+kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream);
+
+/* Depth profile of Eq. 6 on the host: kind 0 Global (lambda = sinh(c[0]) on every
+ * layer), 1 Segments (sinh(c[0]), sinh(c[1]), sinh(c[2]) on layers
+ * [0, b0), [b0, b1), [b1, N_L), with seg_bounds = {b0, b1}, or thirds when
+ * seg_bounds is NULL), 2 Curve (sinh(c0 + c1 t + c2 t^2), t = l / (N_L - 1)).
+ * Writes lambda_out[num_layers]. */
+kve_status kv_evict_profile(int32_t kind, const float* c, int32_t num_layers,
+                            const int32_t* seg_bounds, float* lambda_out);
+
+const char* kv_evict_strerror(kve_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KV_EVICT_H */
