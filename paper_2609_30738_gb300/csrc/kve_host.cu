@@ -1,0 +1,278 @@
+// Host side of the kv_evict C ABI: plan validation and work geometry, workspace
+// layout, TMA descriptor encoding and the launches of the three kernels.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <new>
+
+#include <cudaTypedefs.h>
+
+#include "kve_internal.h"
+
+namespace {
+
+using kve::kHeadDim;
+using kve::kMaxLayers;
+using kve::kMaxReq;
+using kve::kMaxRows;
+using kve::kSplitKeys;
+
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;   // 2 s
+constexpr int kMaxCand = 512;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// [rows][128] bf16 viewed as a 2-D tensor; boxes of 64 elements x 128 rows with the
+// 128-byte swizzle, rows past the end read as zero.
+bool encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(kHeadDim) * 2};
+  cuuint32_t box[2] = {64, 128};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int device_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+}  // namespace
+
+extern "C" {
+
+kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t n_req,
+                         kve_plan** plan_out, size_t* workspace_bytes) {
+  if (!cfg || !seq_lens || !plan_out) return KVE_EINVAL;
+  *plan_out = nullptr;
+  const kve_config& c = *cfg;
+  if (c.num_layers < 1 || c.num_layers > kMaxLayers) return KVE_EINVAL;
+  if (c.num_kv_heads < 1 || c.num_q_heads < c.num_kv_heads || c.num_q_heads % c.num_kv_heads) return KVE_EINVAL;
+  if (c.head_dim != kHeadDim) return KVE_EINVAL;
+  const int G = c.num_q_heads / c.num_kv_heads;
+  if (c.window < 1 || static_cast<int64_t>(G) * c.window > kMaxRows) return KVE_EINVAL;
+  if (c.budget < 1 || c.pool_kernel < 1 || c.pool_kernel % 2 == 0) return KVE_EINVAL;
+  if (c.candidate_factor < 0 || !(c.norm_eps > 0.f) || !std::isfinite(c.norm_eps)) return KVE_EINVAL;
+  if (n_req < 1 || n_req > kMaxReq) return KVE_EINVAL;
+
+  kve_plan* plan = new (std::nothrow) kve_plan;
+  if (!plan) return KVE_ENOMEM;
+  std::memset(plan, 0, sizeof(*plan));
+  plan->cfg = c;
+  plan->wait_limit_ns = kDefaultWaitNs;
+  plan->fault = 0;
+  kve::Geometry& g = plan->geo;
+  g.n_req = n_req;
+  g.num_layers = c.num_layers;
+  g.hq = c.num_q_heads;
+  g.hkv = c.num_kv_heads;
+  g.group = G;
+  g.window = c.window;
+  g.n_rows = G * c.window;
+  int64_t off = 0, units = 0, items = 0, max_lc = 0;
+  const int64_t units_per_req = static_cast<int64_t>(c.num_layers) * c.num_kv_heads;
+  for (int r = 0; r < n_req; ++r) {
+    const int64_t L = seq_lens[r];
+    if (L <= c.window || L > (int64_t(1) << 30)) {
+      delete plan;
+      return KVE_EINVAL;
+    }
+    g.req_len[r] = static_cast<int32_t>(L);
+    g.req_tok_off[r] = off;
+    g.req_splits[r] = static_cast<int32_t>((L + kSplitKeys - 1) / kSplitKeys);
+    g.req_unit_base[r] = units;
+    g.req_item_base[r] = items;
+    off += L;
+    units += units_per_req;
+    items += units_per_req * g.req_splits[r];
+    if (L - c.window > max_lc) max_lc = L - c.window;
+  }
+  g.req_unit_base[n_req] = units;
+  g.req_item_base[n_req] = items;
+  g.total_tokens = off;
+  g.n_units = units;
+  g.n_items = items;
+  const int64_t max_cand = c.candidate_factor == 0 ? max_lc
+                                                   : std::min<int64_t>(int64_t(c.candidate_factor) * c.budget, max_lc);
+  // TMA row coordinates are 32-bit; the select kernel holds its pool in shared memory
+  const int64_t k_rows = units_per_req * off;
+  const int64_t q_rows = static_cast<int64_t>(c.num_layers) * n_req * c.num_q_heads * c.window;
+  if (max_cand > kMaxCand || k_rows >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
+      2 * items >= (int64_t(1) << 31) || units >= (int64_t(1) << 31)) {
+    delete plan;
+    return KVE_EINVAL;
+  }
+  kve::WsLayout& w = plan->ws;
+  w.hdr = 0;
+  w.counts = 256;
+  w.flags = align_up(w.counts + 4 * units, 256);
+  w.clear_end = align_up(w.flags + 4 * units, 256);
+  w.partial = w.clear_end;
+  w.beta = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
+  w.keys = align_up(w.beta + sizeof(float) * kMaxRows * units, 256);
+  w.total = align_up(w.keys + sizeof(uint32_t) * units_per_req * off, 256);
+  if (workspace_bytes) *workspace_bytes = w.total;
+  *plan_out = plan;
+  return KVE_OK;
+}
+
+void kv_evict_plan_destroy(kve_plan* plan) { delete plan; }
+
+kve_status kv_evict_plan_set_debug(kve_plan* plan, uint64_t wait_limit_ns, int32_t fault) {
+  if (!plan || wait_limit_ns == 0 || fault < 0 || fault > 1) return KVE_EINVAL;
+  plan->wait_limit_ns = wait_limit_ns;
+  plan->fault = fault;
+  return KVE_OK;
+}
+
+kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, float* mu,
+                          float* sigma, void* ws, void* stream) {
+  if (!plan || !q_win || !k || !mu || !sigma || !ws) return KVE_EINVAL;
+  if (!aligned(q_win, 128) || !aligned(k, 128) || !aligned(mu, 16) || !aligned(sigma, 16) || !aligned(ws, 256))
+    return KVE_EINVAL;
+  const kve::Geometry& g = plan->geo;
+  const int sms = device_sms();
+  if (sms <= 0) return KVE_ECUDA;
+  CUtensorMap tm_q, tm_k;
+  const int64_t q_rows = static_cast<int64_t>(g.num_layers) * g.n_req * g.hq * g.window;
+  const int64_t k_rows = static_cast<int64_t>(g.num_layers) * g.hkv * g.total_tokens;
+  if (!encode_rows(&tm_q, q_win, q_rows) || !encode_rows(&tm_k, k, k_rows)) return KVE_ECUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  if (cudaMemsetAsync(w, 0, plan->ws.clear_end, st) != cudaSuccess) return KVE_ECUDA;
+  kve::ScoreParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.alpha = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
+  int max_splits = 1;
+  for (int r = 0; r < g.n_req; ++r) max_splits = std::max(max_splits, g.req_splits[r]);
+  p.lag = std::min<int64_t>(g.n_items, static_cast<int64_t>(max_splits) + 2 * sms);
+  p.wait_limit_ns = plan->wait_limit_ns;
+  p.fault = plan->fault;
+  p.mu = mu;
+  p.sigma = sigma;
+  p.err = reinterpret_cast<uint32_t*>(w);
+  p.claim = reinterpret_cast<uint32_t*>(w + 4);
+  p.counts = reinterpret_cast<uint32_t*>(w + plan->ws.counts);
+  p.flags = reinterpret_cast<uint32_t*>(w + plan->ws.flags);
+  p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
+  p.beta = reinterpret_cast<float*>(w + plan->ws.beta);
+  return kve::launch_score(*plan, tm_q, tm_k, p, sms, st) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}
+
+kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
+                           const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
+                           float* margins, void* ws, void* stream) {
+  if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws) return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
+  const kve::Geometry& g = plan->geo;
+  kve::SelectParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.budget = plan->cfg.budget;
+  p.pool_kernel = plan->cfg.pool_kernel;
+  p.cand_factor = plan->cfg.candidate_factor;
+  p.norm_eps = plan->cfg.norm_eps;
+  for (int l = 0; l < g.num_layers; ++l) {
+    if (!std::isfinite(lambda1[l]) || !std::isfinite(lambda2[l])) return KVE_EINVAL;
+    p.lambda1[l] = lambda1[l];
+    p.lambda2[l] = lambda2[l];
+  }
+  p.mu = mu;
+  p.sigma = sigma;
+  p.k = k;
+  p.indices = indices;
+  p.order = order;
+  p.margins = margins;
+  p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.keys);
+  return kve::launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}
+
+kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16_t* v, const int32_t* indices,
+                           uint16_t* k_out, uint16_t* v_out, void* stream) {
+  if (!plan || !k || !v || !indices || !k_out || !v_out) return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(v, 16) || !aligned(k_out, 16) || !aligned(v_out, 16)) return KVE_EINVAL;
+  kve::GatherParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.g = plan->geo;
+  p.budget = plan->cfg.budget;
+  p.k = k;
+  p.v = v;
+  p.indices = indices;
+  p.k_out = k_out;
+  p.v_out = v_out;
+  return kve::launch_gather(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}
+
+kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream) {
+  if (!plan || !ws) return KVE_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return KVE_ECUDA;
+  uint32_t err = 0;
+  if (cudaMemcpy(&err, ws, sizeof(err), cudaMemcpyDeviceToHost) != cudaSuccess) return KVE_ECUDA;
+  if (err != 0) {
+    if (cudaMemset(ws, 0, sizeof(err)) != cudaSuccess) return KVE_ECUDA;
+    return KVE_ETIMEOUT;
+  }
+  return KVE_OK;
+}
+
+kve_status kv_evict_profile(int32_t kind, const float* c, int32_t num_layers, const int32_t* seg_bounds,
+                            float* lambda_out) {
+  if (!c || !lambda_out || num_layers < 1 || kind < 0 || kind > 2) return KVE_EINVAL;
+  int b0 = (num_layers + 2) / 3, b1 = (2 * num_layers + 2) / 3;   // ceil(N/3), ceil(2N/3)
+  if (seg_bounds) {
+    b0 = seg_bounds[0];
+    b1 = seg_bounds[1];
+    if (b0 < 0 || b1 < b0 || b1 > num_layers) return KVE_EINVAL;
+  }
+  for (int l = 0; l < num_layers; ++l) {
+    double a;
+    if (kind == 0) {
+      a = c[0];
+    } else if (kind == 1) {
+      a = l < b0 ? c[0] : (l < b1 ? c[1] : c[2]);
+    } else {
+      const double t = num_layers > 1 ? static_cast<double>(l) / (num_layers - 1) : 0.0;
+      a = static_cast<double>(c[0]) + static_cast<double>(c[1]) * t + static_cast<double>(c[2]) * t * t;
+    }
+    lambda_out[l] = static_cast<float>(std::sinh(a));
+  }
+  return KVE_OK;
+}
+
+const char* kv_evict_strerror(kve_status s) {
+  switch (s) {
+    case KVE_OK: return "ok";
+    case KVE_EINVAL: return "invalid argument or unsupported shape";
+    case KVE_ECUDA: return "CUDA call failed";
+    case KVE_ETIMEOUT: return "device-side wait timed out";
+    case KVE_ENOMEM: return "host allocation failed";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

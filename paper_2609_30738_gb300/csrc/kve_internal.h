@@ -1,0 +1,143 @@
+// Internal declarations of the kv_evict library: the host plan, kernel parameter
+// blocks and the unit / work-item geometry shared by host and device code.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "../../include/kv_evict.h"
+
+namespace kve {
+
+constexpr int kHeadDim = 128;      // d supported by this build
+constexpr int kTileKeys = 128;     // keys per MMA tile (one TMEM accumulator)
+constexpr int kSplitTiles = 4;     // tiles per work item
+constexpr int kSplitKeys = kTileKeys * kSplitTiles;
+constexpr int kMaxRows = 128;      // n = G*W window rows per unit, padded to one M tile
+constexpr int kMaxReq = 64;        // requests per call
+constexpr int kMaxLayers = 256;    // layers per call (lambda arrays ride in kernel params)
+
+// Request table and derived counts, identical on host and device.
+struct Geometry {
+  int32_t n_req, num_layers, hq, hkv, group, window, n_rows;
+  int64_t total_tokens;                 // SL
+  int64_t n_units;                      // n_req * N_L * Hkv
+  int64_t n_items;                      // score work items (sum over units of splits)
+  int32_t req_len[kMaxReq];             // L_r
+  int64_t req_tok_off[kMaxReq];         // off_r
+  int32_t req_splits[kMaxReq];          // ceil(L_r / kSplitKeys)
+  int64_t req_unit_base[kMaxReq + 1];   // first unit of request r
+  int64_t req_item_base[kMaxReq + 1];   // first item of request r
+};
+
+struct UnitInfo {
+  int64_t unit;        // (r, l, h) flattened, request-major
+  int32_t r, layer, h;
+  int32_t L;           // prefix length
+  int32_t splits;      // items of this unit
+  int64_t q_row0;      // first window row in q_win viewed as [rows][d]
+  int64_t k_row0;      // first key row in k viewed as [rows][d]
+  int64_t mu_off;      // first element of this unit in mu / sigma
+  int64_t item0;       // first score item of this unit
+};
+
+__host__ __device__ inline UnitInfo unit_info(const Geometry& g, int64_t unit) {
+  int r = 0;
+  while (r + 1 < g.n_req && g.req_unit_base[r + 1] <= unit) ++r;
+  UnitInfo u;
+  u.unit = unit;
+  u.r = r;
+  const int64_t local = unit - g.req_unit_base[r];
+  u.layer = static_cast<int32_t>(local / g.hkv);
+  u.h = static_cast<int32_t>(local % g.hkv);
+  u.L = g.req_len[r];
+  u.splits = g.req_splits[r];
+  u.q_row0 = ((static_cast<int64_t>(u.layer) * g.n_req + r) * g.hq +
+              static_cast<int64_t>(u.h) * g.group) * g.window;
+  u.k_row0 = (static_cast<int64_t>(u.layer) * g.hkv + u.h) * g.total_tokens + g.req_tok_off[r];
+  u.mu_off = static_cast<int64_t>(g.num_layers) * g.hkv * g.req_tok_off[r] + local * u.L;
+  u.item0 = g.req_item_base[r] + local * u.splits;
+  return u;
+}
+
+// Score item p (0 <= p < n_items) -> unit and split index.
+__host__ __device__ inline int64_t item_unit(const Geometry& g, int64_t p, int32_t* split) {
+  int r = 0;
+  while (r + 1 < g.n_req && g.req_item_base[r + 1] <= p) ++r;
+  const int64_t local = p - g.req_item_base[r];
+  *split = static_cast<int32_t>(local % g.req_splits[r]);
+  return g.req_unit_base[r] + local / g.req_splits[r];
+}
+
+// Workspace layout (byte offsets from the caller's workspace pointer).
+struct WsLayout {
+  size_t hdr;        // uint32 err, uint32 claim, padding to 256 B
+  size_t counts;     // uint32 [n_units]  row-statistics arrivals per unit
+  size_t flags;      // uint32 [n_units]  merged statistics ready
+  size_t clear_end;  // bytes from 0 cleared before each score call
+  size_t partial;    // float2 [n_items][kMaxRows]  per-item (max, sum) in log2 units
+  size_t beta;       // float  [n_units][kMaxRows]  log2 softmax normaliser per row
+  size_t keys;       // uint32 [sum of unit lengths]  ordered base scores (select)
+  size_t total;
+};
+
+struct ScoreParams {
+  Geometry g;
+  float alpha;               // log2(e) / sqrt(d)
+  int64_t lag;               // row-statistics items issued before the first column item
+  uint64_t wait_limit_ns;
+  int32_t fault;             // test hook: 1 = unit 0 never publishes its statistics
+  float* mu;
+  float* sigma;
+  uint32_t* err;
+  uint32_t* claim;
+  uint32_t* counts;
+  uint32_t* flags;
+  float2* partial;
+  float* beta;
+};
+
+struct SelectParams {
+  Geometry g;
+  int32_t budget, pool_kernel, cand_factor;
+  float norm_eps;
+  const float* mu;
+  const float* sigma;
+  const uint16_t* k;
+  int32_t* indices;
+  int32_t* order;
+  float* margins;
+  uint32_t* keys;            // workspace scratch
+  float lambda1[kMaxLayers];
+  float lambda2[kMaxLayers];
+};
+
+struct GatherParams {
+  Geometry g;
+  int32_t budget;
+  const uint16_t* k;
+  const uint16_t* v;
+  const int32_t* indices;
+  uint16_t* k_out;
+  uint16_t* v_out;
+};
+
+}  // namespace kve
+
+struct kve_plan {
+  kve_config cfg;
+  kve::Geometry geo;
+  kve::WsLayout ws;
+  uint64_t wait_limit_ns;
+  int32_t fault;
+};
+
+namespace kve {
+// Kernel launchers (defined next to their kernels).
+cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                         const ScoreParams& p, int num_sms, cudaStream_t stream);
+cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
+cudaError_t launch_gather(const kve_plan& plan, const GatherParams& p, cudaStream_t stream);
+}  // namespace kve

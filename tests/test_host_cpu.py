@@ -1,0 +1,85 @@
+"""Host-side checks that need no GPU: the library loads and exports every entry
+point of include/kv_evict.h, plan validation and the Eq. 6 profile helper."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import kv_evict_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+LIB = os.path.join(ROOT, "paper_2609_30738_gb300", "libkvevict.so")
+
+
+def _need_lib():
+    if not os.path.exists(LIB):
+        pytest.skip("library not built")
+
+
+def _spec(**over):
+    s = dict(num_layers=2, num_q_heads=32, num_kv_heads=8, head_dim=128, window=32, budget=64,
+             pool_kernel=7, candidate_factor=4, norm_eps=1e-12)
+    s.update(over)
+    return s
+
+
+def test_header_symbols_are_exported():
+    _need_lib()
+    header = open(os.path.join(ROOT, "include", "kv_evict.h")).read()
+    names = set(re.findall(r"\b(kv_evict_\w+)\s*\(", header))
+    assert len(names) >= 9
+    lib = ctypes.CDLL(LIB)
+    for n in sorted(names):
+        assert hasattr(lib, n), n
+    from paper_2609_30738_gb300 import kv_evict as K
+    assert names == set(K.EXPORTS)
+
+
+def test_plan_sizes_and_validation():
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    p = K.Plan(_spec(), [2048, 777])
+    assert p.n_units == 2 * 2 * 8
+    assert p.score_elems == 2 * 8 * (2048 + 777)
+    assert p.workspace_bytes > 0 and p.workspace_bytes % 256 == 0
+    bad = [
+        (_spec(head_dim=64), [100]),          # d != 128
+        (_spec(window=33), [100]),            # G*W > 128
+        (_spec(num_q_heads=30), [100]),       # Hq not a multiple of Hkv
+        (_spec(pool_kernel=4), [100]),        # even pooling kernel
+        (_spec(budget=0), [100]),
+        (_spec(budget=200), [5000]),          # 4B > 512 candidates
+        (_spec(), [32]),                      # L <= W
+        (_spec(norm_eps=0.0), [100]),
+        (_spec(num_layers=0), [100]),
+        (_spec(), [100] * 65),                # too many requests
+    ]
+    for spec, lens in bad:
+        with pytest.raises(K.KvEvictError) as e:
+            K.Plan(spec, lens)
+        assert e.value.status == K.KVE_EINVAL
+
+
+def test_null_arguments_rejected_without_gpu():
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    lib = K.library()
+    p = K.Plan(_spec(), [300])
+    assert lib.kv_evict_score(p._h, None, None, None, None, None, None) == K.KVE_EINVAL
+    assert lib.kv_evict_gather(None, None, None, None, None, None, None) == K.KVE_EINVAL
+    assert lib.kv_evict_plan_set_debug(p._h, 0, 0) == K.KVE_EINVAL
+    assert lib.kv_evict_strerror(K.KVE_ETIMEOUT) == b"device-side wait timed out"
+
+
+@pytest.mark.parametrize("kind,c", [("global", [0.3]), ("segments", [-0.8, 0.6, -0.8]),
+                                    ("curve", [0.1, -0.7, 1.3])])
+@pytest.mark.parametrize("N", [1, 5, 32])
+def test_profile_matches_oracle(kind, c, N):
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    lib_vals = K.profile(kind, c, N)
+    ref = O.depth_profile(kind, c, N)
+    np.testing.assert_allclose(lib_vals, ref, rtol=2e-7, atol=1e-7)

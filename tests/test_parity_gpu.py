@@ -1,0 +1,213 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle. GPU only."""
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from oracle import kv_evict_oracle as O
+from paper_2609_30738_gb300 import synth
+from paper_2609_30738_gb300.workloads import WORKLOADS, lambda_arrays, scaled
+
+from tests import parity as PT
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2609_30738_gb300 import kv_evict as K
+    K.library()   # fails loudly when the library is missing
+    return K
+
+
+def _run(spec, batch, lambdas=None):
+    from paper_2609_30738_gb300 import kv_evict as K
+    plan = K.Plan(spec, batch["seq_lens"])
+    bufs = K.Buffers(plan)
+    if lambdas is None:
+        lambdas = lambda_arrays(spec, K.profile)
+    q, k, v = (batch[x].to(DEV) for x in ("q_win", "k", "v"))
+    K.run_step(plan, bufs, q, k, v, lambdas[0], lambdas[1])
+    assert plan.status(bufs.ws) == K.KVE_OK
+    return plan, bufs, (q, k, v), lambdas
+
+
+def _unit_index(spec, seq_lens, r, layer, h):
+    return (r * spec["num_layers"] + layer) * spec["num_kv_heads"] + h
+
+
+def _mu_offset(spec, seq_lens, r, layer, h):
+    N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
+    return N_L * Hkv * sum(seq_lens[:r]) + (layer * Hkv + h) * seq_lens[r]
+
+
+def _check_units(spec, batch, plan, bufs, lambdas, units, sel_mode="replay"):
+    """Oracle comparison of the listed units (r, layer, h). Returns max mu rel error
+    and the list of near-tie swaps."""
+    seq = batch["seq_lens"]
+    W, B, G = spec["window"], spec["budget"], spec["num_q_heads"] // spec["num_kv_heads"]
+    mu_all = bufs.mu.cpu().numpy()
+    sg_all = bufs.sigma.cpu().numpy()
+    idx_all = bufs.indices.cpu().numpy()
+    ord_all = bufs.order.cpu().numpy()
+    mar_all = bufs.margins.cpu().numpy()
+    worst, swaps = 0.0, []
+    for (r, layer, h) in units:
+        L = seq[r]
+        off = sum(seq[:r])
+        qb = PT.to_bits(batch["q_win"][layer, r, h * G:(h + 1) * G]).reshape(G * W, -1)
+        kb = PT.to_bits(batch["k"][layer, h, off:off + L])
+        vb = PT.to_bits(batch["v"][layer, h, off:off + L])
+        qf, kf = O.bf16_bits_to_f64(qb), O.bf16_bits_to_f64(kb)
+        mu_ref, sg_ref = O.score_unit(qf, kf, L, W, G)
+        o = _mu_offset(spec, seq, r, layer, h)
+        tag = f"unit(r={r},l={layer},h={h})"
+        worst = max(worst, PT.check_mu_sigma(mu_all[o:o + L], sg_all[o:o + L], mu_ref, sg_ref, tag))
+        ui = _unit_index(spec, seq, r, layer, h)
+        swaps += PT.check_selection(ord_all[ui], idx_all[ui], mu_ref, sg_ref, kf, L, W, B,
+                                    float(lambdas[0][layer]), float(lambdas[1][layer]),
+                                    spec["pool_kernel"], spec["candidate_factor"],
+                                    spec["norm_eps"], margins_gpu=mar_all[ui], what=tag)
+        ko = PT.to_bits(bufs.k_out[ui])
+        vo = PT.to_bits(bufs.v_out[ui])
+        PT.check_gather(ko, vo, kb, vb, idx_all[ui], L, W, B)
+    return worst, swaps
+
+
+def _all_units(spec, seq):
+    return [(r, l, h) for r in range(len(seq)) for l in range(spec["num_layers"])
+            for h in range(spec["num_kv_heads"])]
+
+
+# ---------------------------------------------------------------- small cases, every unit
+
+
+def test_single_layer_L2048_every_unit():
+    spec = WORKLOADS["mistral-1layer-L2048"]
+    batch = synth.make_batch(spec, seed=2609)
+    plan, bufs, _, lam = _run(spec, batch)
+    worst, swaps = _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+    print(f"max mu rel err {worst:.2e}, near-tie swaps {swaps}")
+
+
+def test_ragged_requests_and_tails():
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=16,
+                  seq_lens=[300, 777, 1500, 40, 513])
+    batch = synth.make_batch(spec, seed=7)
+    plan, bufs, _, lam = _run(spec, batch)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
+def test_window8_partial_rows():
+    """W = 8 as in the paper: n = 32 window rows per KV head."""
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], window=8, budget=32, seq_lens=[1000, 129])
+    batch = synth.make_batch(spec, seed=8)
+    plan, bufs, _, lam = _run(spec, batch)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
+@pytest.mark.parametrize("lams", [(0.0, 0.0), (0.0, -0.15), (0.5, 0.6), (-0.3, -0.5), (2.0, -3.6)])
+def test_lambda_settings(lams):
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[1200], lambdas=("global",) + lams)
+    batch = synth.make_batch(spec, seed=9)
+    plan, bufs, _, lam = _run(spec, batch)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
+def test_lambda_zero_is_mean_attention_topB():
+    """lambda1 = lambda2 = 0: the kept set is the top-B of pooled mean attention."""
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[1500], lambdas=("global", 0.0, 0.0))
+    batch = synth.make_batch(spec, seed=10)
+    plan, bufs, _, lam = _run(spec, batch)
+    mu = bufs.mu.cpu().numpy()
+    idx = bufs.indices.cpu().numpy()
+    L, W, B = 1500, spec["window"], spec["budget"]
+    for h in range(spec["num_kv_heads"]):
+        o = h * L
+        pooled = O.max_pool(mu[o:o + L - W].astype(np.float64), spec["pool_kernel"])
+        ref = np.sort(O.rank_desc(pooled)[:B])
+        assert np.array_equal(idx[h], ref)
+
+
+@pytest.mark.parametrize("L,B,pk,cf", [(33, 64, 7, 4), (40, 64, 7, 4), (100, 64, 7, 4),
+                                       (129, 8, 1, 4), (512, 16, 5, 4), (544, 32, 7, 0),
+                                       (1025, 128, 3, 4), (4097, 64, 7, 2)])
+def test_edge_shapes(L, B, pk, cf):
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[L], budget=B, pool_kernel=pk,
+                  candidate_factor=cf)
+    batch = synth.make_batch(spec, seed=L)
+    plan, bufs, _, lam = _run(spec, batch)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
+def test_repeatable_bitwise():
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[3000, 700])
+    batch = synth.make_batch(spec, seed=11)
+    plan, bufs, (q, k, v), lam = _run(spec, batch)
+    mu1, sg1, idx1 = bufs.mu.clone(), bufs.sigma.clone(), bufs.indices.clone()
+    from paper_2609_30738_gb300 import kv_evict as K
+    K.run_step(plan, bufs, q, k, v, lam[0], lam[1])
+    assert torch.equal(mu1, bufs.mu) and torch.equal(sg1, bufs.sigma)
+    assert torch.equal(idx1, bufs.indices)
+
+
+def test_bounded_wait_reports_timeout_and_gpu_stays_usable():
+    """A unit whose row statistics are never published (host-set test hook): the
+    column pass waits out a 5 ms limit, reports KVE_ETIMEOUT, and the next call
+    on the same plan works."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[1024])
+    batch = synth.make_batch(spec, seed=12)
+    plan = K.Plan(spec, batch["seq_lens"])
+    bufs = K.Buffers(plan)
+    q, k = batch["q_win"].to(DEV), batch["k"].to(DEV)
+    plan.set_debug(5_000_000, fault=1)
+    plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws)
+    assert plan.status(bufs.ws) == K.KVE_ETIMEOUT
+    plan.set_debug(2_000_000_000, fault=0)
+    plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws)
+    assert plan.status(bufs.ws) == K.KVE_OK
+    kb = PT.to_bits(batch["k"][0, 0, :1024])
+    qb = PT.to_bits(batch["q_win"][0, 0, 0:4]).reshape(128, -1)
+    mu_ref, sg_ref = O.score_unit(O.bf16_bits_to_f64(qb), O.bf16_bits_to_f64(kb), 1024, 32, 4)
+    PT.check_mu_sigma(bufs.mu[:1024].cpu().numpy(), bufs.sigma[:1024].cpu().numpy(), mu_ref, sg_ref)
+
+
+# ---------------------------------------------------------------- full-size workloads, sampled units
+
+
+FULL = ["mistral-32layer-L8192", "mistral-32layer-L32768-B32", "mistral-32layer-L32768-B64",
+        "mistral-32layer-L32768-B128", "mistral-32layer-L16384-segments", "mistral-32layer-ragged16"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled_units(name):
+    spec = WORKLOADS[name]
+    batch = synth.make_batch(spec, seed=2609, device=DEV)
+    plan, bufs, _, lam = _run(spec, batch)
+    seq = batch["seq_lens"]
+    N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
+    # properties on every unit: each unit's mu sums to 1 (every row is a distribution)
+    sums = []
+    off = 0
+    for r, L in enumerate(seq):
+        seg = bufs.mu[N_L * Hkv * off: N_L * Hkv * (off + L)].view(N_L * Hkv, L).double().sum(1)
+        sums.append(seg)
+        off += L
+    sums = torch.cat(sums)
+    assert torch.all((sums - 1).abs() < 1e-3), float((sums - 1).abs().max())
+    idx = bufs.indices
+    B = spec["budget"]
+    assert torch.all(idx[:, 1:] > idx[:, :-1]), "indices ascending and unique"
+    # oracle on sampled units: first, last, middle layer; shortest and longest request
+    r_lo = int(np.argmin(seq))
+    r_hi = int(np.argmax(seq))
+    units = sorted({(0, 0, 0), (r_hi, N_L - 1, Hkv - 1), (r_lo, N_L // 2, 3), (r_hi, 11, 5),
+                    (len(seq) - 1, 21, 2)})
+    worst, swaps = _check_units(spec, batch, plan, bufs, lam, units)
+    print(f"{name}: max mu rel err {worst:.2e}, near-tie swaps {swaps}")
