@@ -1,0 +1,444 @@
+"""Benchmark of the end-of-prefill diversified KV-eviction step on GB300.
+
+One step = the whole path for one request of the Mistral-7B-shaped workload
+"mistral-32layer-L32768-B64": 32 layers x 8 KV heads (256 units), prefix 32768,
+window 32, budget 64, lambda = (0.5, -0.5): score (window attention, mu, sigma),
+select (pooling, top-4B, greedy MMR) and gather (compact K/V cache).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+N > 1 runs under torchrun, one rank per GPU; every rank evicts its own request
+(weak scaling, no collective on the data path). Rank 0 prints one JSON line.
+--impl reference times the fp64 CPU oracle (the only reference this path has) on
+a bounded sample of the same workload on the host cores.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "mistral-32layer-L32768-B64"
+METRIC = "eviction-step ms/request (32 layers) & prefix tok/s; % of HBM roofline"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+
+# DRAM traffic of one score-kernel launch (dram__bytes_read.sum + dram__bytes_write.sum),
+# from the ncu capture summarised in profiles/, valid only for the kernel source it was
+# taken on (sha256 of csrc/kve_score.cu); per launch of the full workload.
+SCORE_TRAFFIC = {"source_sha256": None, "bytes_per_launch": None}
+
+
+def _score_source_sha():
+    p = os.path.join(ROOT, "paper_2609_30738_gb300", "csrc", "kve_score.cu")
+    return hashlib.sha256(open(p, "rb").read()).hexdigest()
+
+
+def _peaks():
+    try:
+        d = json.load(open(PEAKS_FILE))
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "50", "-i", str(self.gpu)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def mark(self, which):
+        setattr(self, which, time.time())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        rows = [r.split(", ") for r in out.strip().splitlines() if r.strip()]
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+                for nm, val in zip(names, r[5:9]):
+                    if val.strip().lower() == "active":
+                        reasons.add(nm)
+            except (ValueError, IndexError):
+                continue
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ oracle baseline
+
+
+_SAMPLE = None
+
+
+def _oracle_init(path, n_units, q_shape, k_shape, meta):
+    """Worker initialiser: map the shared sample file (no copies per task)."""
+    global _SAMPLE
+    qn = int(np.prod(q_shape))
+    kn = int(np.prod(k_shape))
+    mm = np.memmap(path, dtype=np.uint16, mode="r", shape=(n_units, qn + kn))
+    _SAMPLE = (mm, q_shape, k_shape, meta)
+
+
+def _oracle_unit(u):
+    """Score and select one unit with the fp64 oracle (runs in a spawned worker)."""
+    from oracle import kv_evict_oracle as O
+    mm, q_shape, k_shape, (L, W, G, B, l1, l2) = _SAMPLE
+    qn = int(np.prod(q_shape))
+    q_bits = np.asarray(mm[u, :qn]).reshape(q_shape)
+    k_bits = np.asarray(mm[u, qn:]).reshape(k_shape)
+    t = time.perf_counter()
+    O.evict_unit(q_bits, k_bits, L, W, G, B, l1, l2)
+    return time.perf_counter() - t
+
+
+class OraclePool:
+    """Spawned worker processes (one BLAS thread each) over a memory-mapped sample."""
+
+    def __init__(self, spec, sample, workers):
+        import multiprocessing as mp
+        import tempfile
+        for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+            os.environ[var] = "1"
+        G = spec["num_q_heads"] // spec["num_kv_heads"]
+        q_shape, k_shape = sample[0][0].shape, sample[0][1].shape
+        self.dir = tempfile.mkdtemp(prefix="kve_oracle_")
+        self.path = os.path.join(self.dir, "sample.u16")
+        n = len(sample)
+        mm = np.memmap(self.path, dtype=np.uint16, mode="w+",
+                       shape=(n, int(np.prod(q_shape)) + int(np.prod(k_shape))))
+        for i, (q, k) in enumerate(sample):
+            mm[i] = np.concatenate([q.reshape(-1), k.reshape(-1)])
+        mm.flush()
+        del mm
+        meta = (spec["seq_lens"][0], spec["window"], G, spec["budget"], 0.5, -0.5)
+        self.n = n
+        self.pool = mp.get_context("spawn").Pool(
+            workers, initializer=_oracle_init, initargs=(self.path, n, q_shape, k_shape, meta))
+
+    def run(self):
+        """Wall time of one pass over every unit of the sample."""
+        t = time.perf_counter()
+        self.pool.map(_oracle_unit, range(self.n), chunksize=1)
+        return time.perf_counter() - t
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+        try:
+            os.remove(self.path)
+            os.rmdir(self.dir)
+        except OSError:
+            pass
+
+
+def _oracle_sample_from_host(spec, n_units, seed):
+    """(q_bits, k_bits) of the first n_units units, generated on the CPU."""
+    import torch
+    from paper_2609_30738_gb300 import synth
+    from tests.parity import to_bits
+    G = spec["num_q_heads"] // spec["num_kv_heads"]
+    W, L, Hkv = spec["window"], spec["seq_lens"][0], spec["num_kv_heads"]
+    out = []
+    layer = 0
+    while len(out) < n_units:
+        k, v, q = synth.unit_tensors(seed, 0, layer, L, Hkv, G, W,
+                                     salient_frac=spec.get("salient_frac", 0.0))
+        for h in range(Hkv):
+            if len(out) < n_units:
+                out.append((to_bits(q[h].to(torch.bfloat16)), to_bits(k[h].to(torch.bfloat16))))
+        layer += 1
+    return out
+
+
+def run_reference(args):
+    """--impl reference: the fp64 oracle on the host cores, bounded sample per step."""
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    from paper_2609_30738_gb300.workloads import WORKLOADS
+    spec = WORKLOADS[WORKLOAD]
+    cores = os.cpu_count() or 1
+    n_units = cores          # one unit per host core and step
+    sample = _oracle_sample_from_host(spec, n_units, 2609)
+    pool = OraclePool(spec, sample, cores)
+    try:
+        for _ in range(args.warmup):
+            pool.run()
+        times = [pool.run() for _ in range(args.steps)]
+    finally:
+        pool.close()
+    step_s = sum(times) / len(times)
+    units_total = spec["num_layers"] * spec["num_kv_heads"]
+    L = spec["seq_lens"][0]
+    tok_s = L * (n_units / units_total) / step_s
+    ms_req = step_s * 1e3 * units_total / n_units
+    line = {"impl": "reference", "metric": METRIC, "value": tok_s, "unit": "prefix tok/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms_req, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "sample_units": n_units},
+            "cpu_baseline": {"value": tok_s, "unit": "prefix tok/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{n_units} of 256 units (score + select) per step, "
+                                       "extrapolated to the 256-unit request"},
+            "e2e": {"value": tok_s, "unit": "prefix tok/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ GPU arm
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_30738_gb300 import kv_evict as K
+    from paper_2609_30738_gb300 import synth
+    from paper_2609_30738_gb300.workloads import WORKLOADS, lambda_arrays
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    spec = WORKLOADS[WORKLOAD]
+    if args.layers:
+        spec = dict(spec, num_layers=args.layers)
+    L = spec["seq_lens"][0]
+    W, B, d = spec["window"], spec["budget"], spec["head_dim"]
+    N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
+    units = N_L * Hkv
+
+    # inputs resident in HBM: each rank evicts its own request (seeded by rank)
+    batch = synth.make_batch(spec, seed=2609 + rank, device=dev)
+    q, k, v = batch["q_win"], batch["k"], batch["v"]
+    plan = K.Plan(spec, batch["seq_lens"])
+    bufs = K.Buffers(plan, device=dev, with_trace=False)
+    lam1, lam2 = lambda_arrays(spec, K.profile)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step():
+        K.run_step(plan, bufs, q, k, v, lam1, lam2, stream=stream)
+
+    # correctness of the timed configuration: device status after a first step
+    with torch.cuda.stream(stream):
+        step()
+    if plan.status(bufs.ws, stream) != K.KVE_OK:
+        raise RuntimeError("device-side wait timed out")
+
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark("t0")
+    t0.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws, stream)
+        ev[i][1].record(stream)
+        plan.select(bufs.mu, bufs.sigma, k, lam1, lam2, bufs.indices, bufs.ws, None, None, stream)
+        plan.gather(k, v, bufs.indices, bufs.k_out, bufs.v_out, stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark("t1")
+    if world > 1:
+        dist.barrier()
+    elapsed = t0.elapsed_time(t1) / 1e3
+    score_s = sum(a.elapsed_time(b) for a, b in ev) / 1e3 / args.steps
+    clocks = sampler.stop() if sampler else None
+    if plan.status(bufs.ws, stream) != K.KVE_OK:
+        raise RuntimeError("device-side wait timed out in the timed region")
+    if world > 1:
+        t = torch.tensor([elapsed], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed = float(t.item())
+
+    # end to end through the public API with host buffers (pinned), copies inside
+    e2e = None
+    if args.e2e_steps > 0:
+        hq = q.cpu().pin_memory()
+        hk = k.cpu().pin_memory()
+        hv = v.cpu().pin_memory()
+        o_idx = torch.empty_like(bufs.indices, device="cpu").pin_memory()
+        o_k = torch.empty_like(bufs.k_out, device="cpu").pin_memory()
+        o_v = torch.empty_like(bufs.v_out, device="cpu").pin_memory()
+        dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+
+        def e2e_step():
+            with torch.cuda.stream(stream):
+                dq.copy_(hq, non_blocking=True)
+                dk.copy_(hk, non_blocking=True)
+                dv.copy_(hv, non_blocking=True)
+            K.run_step(plan, bufs, dq, dk, dv, lam1, lam2, stream=stream)
+            with torch.cuda.stream(stream):
+                o_idx.copy_(bufs.indices, non_blocking=True)
+                o_k.copy_(bufs.k_out, non_blocking=True)
+                o_v.copy_(bufs.v_out, non_blocking=True)
+
+        e2e_step()
+        stream.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        if world > 1:
+            dist.barrier()
+        a.record(stream)
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        e2e_s = a.elapsed_time(b) / 1e3 / args.e2e_steps
+        if world > 1:
+            t = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t.item())
+        h2d = sum(x.numel() * x.element_size() for x in (hq, hk, hv))
+        d2h = sum(x.numel() * x.element_size() for x in (o_idx, o_k, o_v))
+        e2e = {"value": world * L / e2e_s, "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3}
+        del hq, hk, hv, dq, dk, dv
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    # roofline of the dominant kernel (score): algorithmic bytes per launch
+    n_rows = spec["num_q_heads"] // Hkv * W
+    score_bytes = units * (L * d * 2 + n_rows * d * 2 + 2 * 4 * L)
+    gather_bytes = units * 2 * 2 * (B + W) * d * 2
+    peak, peak_kind = _peaks()
+    achieved = score_bytes / score_s / 1e9
+    traffic = (SCORE_TRAFFIC["bytes_per_launch"]
+               if SCORE_TRAFFIC["source_sha256"] == _score_source_sha() else None)
+
+    cpu = None
+    if world == 1 and args.cpu_units > 0:
+        cpu = cpu_baseline_from_device(spec, batch, args.cpu_units)
+
+    step_s = elapsed / args.steps
+    line = {"metric": METRIC, "value": world * L / step_s, "unit": "prefix tok/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16xbf16->f32", "data": "synthetic (seeded Mistral-7B-shaped K/V/Q)",
+            "config": {"workload": WORKLOAD if not args.layers else f"{WORKLOAD} ({N_L} layers)",
+                       "layers": N_L, "kv_heads": Hkv,
+                       "q_heads": spec["num_q_heads"], "head_dim": d, "prefix_len": L,
+                       "window": W, "budget": B, "lambda1": 0.5, "lambda2": -0.5,
+                       "pool_kernel": spec["pool_kernel"], "requests_per_gpu": 1,
+                       "l2": "inputs larger than L2 (2.15 GB of K read per step)"},
+            "ms_per_request": step_s * 1e3,
+            "hbm_roofline_frac_step": (score_bytes + gather_bytes) / step_s / 1e9 / peak,
+            "score_kernel_ms": score_s * 1e3,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic,
+                         "peak_source": peak_kind, "kernel": "kve score_kernel",
+                         "algorithmic_bytes_per_launch": score_bytes},
+            "gpu_launches": 3 * args.steps,
+            "clocks": clocks, "cpu_baseline": cpu, "e2e": e2e}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def cpu_baseline_from_device(spec, batch, n_units):
+    """Oracle on the first n_units units of the device-resident inputs."""
+    from tests.parity import to_bits
+    G = spec["num_q_heads"] // spec["num_kv_heads"]
+    W, Hkv = spec["window"], spec["num_kv_heads"]
+    sample = []
+    for u in range(n_units):
+        layer, h = divmod(u, Hkv)
+        sample.append((to_bits(batch["q_win"][layer, 0, h * G:(h + 1) * G]).reshape(G * W, -1),
+                       to_bits(batch["k"][layer, h])))
+    cores = min(os.cpu_count() or 1, n_units)
+    pool = OraclePool(spec, sample, cores)
+    try:
+        wall = pool.run()
+    finally:
+        pool.close()
+    units_total = spec["num_layers"] * Hkv
+    L = spec["seq_lens"][0]
+    return {"value": L * (n_units / units_total) / wall, "unit": "prefix tok/s", "cores": cores,
+            "kind": "oracle",
+            "sample": f"{n_units} of {units_total} units (score + select), wall {wall:.1f} s on "
+                      f"{cores} worker processes, extrapolated to the whole request"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-units", type=int, default=128)
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling only: fewer layers than the workload (0 = all)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
