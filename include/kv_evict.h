@@ -122,6 +122,28 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu,
                            int32_t* indices, int32_t* order, float* margins,
                            void* ws, void* stream);
 
+/* Step 3 without a workspace. The paper has no counterpart: this entry point
+ * exists for callers that cannot allocate device memory at eviction time --
+ * serving engines that reserve nearly all of HBM for their own KV-cache pool and
+ * hand kernels only pointers into it, or plugin hosts that give a kernel nothing
+ * but its inputs and outputs. It computes exactly what kv_evict_select computes,
+ * with the same arguments except ws; its scratch (4 bytes per prefix token per
+ * unit) is a 16 MiB array compiled into the library, which every GPU that loads
+ * the library keeps reserved until the process exits. It allocates nothing.
+ *  * Returns KVE_EINVAL when N_L * Hkv * SL exceeds 4194304 (16 MiB / 4 B), e.g.
+ *    a 32-layer, 8-KV-head request of more than 16384 tokens.
+ *  * The first call on a device looks up the array's device address on that
+ *    device (cudaGetSymbolAddress); make that first call before any stream
+ *    capture on the device.
+ *  * All calls share the one array and each call overwrites it before reading it.
+ *    Calls whose executions overlap on the GPU (for example on two streams at
+ *    once) race on it and give undefined results; serialise them. */
+kve_status kv_evict_select_noalloc(const kve_plan* plan, const float* mu,
+                                   const float* sigma, const uint16_t* k,
+                                   const float* lambda1, const float* lambda2,
+                                   int32_t* indices, int32_t* order,
+                                   float* margins, void* stream);
+
 /* Step 4: compact cache (Section 1: each layer keeps B entries after prefill;
  * the window tokens are kept as well). Copies key/value rows bit-exactly. */
 kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k,

@@ -16,6 +16,8 @@
 //     both corr(i, {}) and the clamp at 0);
 //  5. write the admitted positions ascending (and optionally in admission order,
 //     with the best-minus-second margin of every admission).
+#include <mutex>
+
 #include "kve_internal.h"
 
 namespace kve {
@@ -295,3 +297,76 @@ cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStrea
 }
 
 }  // namespace kve
+
+// ---------------------------------------------------------------------------
+// Selection without caller-provided scratch.
+//
+// Some callers cannot allocate device memory when they evict: serving engines
+// that reserve nearly all of HBM up front for their own KV-cache pool and hand
+// kernels nothing but pointers into it (a cudaMalloc there fails or breaks the
+// engine's accounting, and it also synchronises the device), or plugin hosts that
+// give a kernel only its input and output buffers. For them the select kernel's
+// one scratch buffer -- the ordered base score of every candidate token -- lives
+// in a fixed array compiled into this library.
+namespace kve {
+namespace {
+
+constexpr size_t kNoAllocScratchWords = size_t(4) << 20;   // 16 MiB of uint32 keys
+
+// Reserved on every GPU that loads the library, for the life of the process.
+static __device__ __align__(256) uint32_t g_select_scratch[kNoAllocScratchWords];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+uint32_t* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_select_scratch on the current device (looked up once per
+// device; in host code the symbol itself is only a host-side stand-in).
+uint32_t* scratch_on_current_device() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess) return nullptr;
+    g_scratch_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  return g_scratch_ptr[dev];
+}
+
+}  // namespace
+}  // namespace kve
+
+extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float* mu, const float* sigma,
+                                              const uint16_t* k, const float* lambda1,
+                                              const float* lambda2, int32_t* indices, int32_t* order,
+                                              float* margins, void* stream) {
+  using namespace kve;
+  if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices) return KVE_EINVAL;
+  const Geometry& g = plan->geo;
+  const size_t words = static_cast<size_t>(g.num_layers) * g.hkv * static_cast<size_t>(g.total_tokens);
+  if (words > kNoAllocScratchWords) return KVE_EINVAL;   // beyond the fixed scratch
+  if ((reinterpret_cast<uintptr_t>(k) & 15u) != 0) return KVE_EINVAL;
+  uint32_t* scratch = scratch_on_current_device();
+  if (!scratch) return KVE_ECUDA;
+  SelectParams p;
+  memset(&p, 0, sizeof(p));
+  p.g = g;
+  p.budget = plan->cfg.budget;
+  p.pool_kernel = plan->cfg.pool_kernel;
+  p.cand_factor = plan->cfg.candidate_factor;
+  p.norm_eps = plan->cfg.norm_eps;
+  for (int l = 0; l < g.num_layers; ++l) {
+    if (!isfinite(lambda1[l]) || !isfinite(lambda2[l])) return KVE_EINVAL;
+    p.lambda1[l] = lambda1[l];
+    p.lambda2[l] = lambda2[l];
+  }
+  p.mu = mu;
+  p.sigma = sigma;
+  p.k = k;
+  p.indices = indices;
+  p.order = order;
+  p.margins = margins;
+  p.keys = scratch;
+  return launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}

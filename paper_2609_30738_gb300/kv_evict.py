@@ -19,8 +19,8 @@ KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 
 # Names declared in include/kv_evict.h.
 EXPORTS = ("kv_evict_plan", "kv_evict_plan_destroy", "kv_evict_plan_set_debug", "kv_evict_score",
-           "kv_evict_select", "kv_evict_gather", "kv_evict_status", "kv_evict_profile",
-           "kv_evict_strerror")
+           "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather", "kv_evict_status",
+           "kv_evict_profile", "kv_evict_strerror")
 
 
 class KvEvictError(RuntimeError):
@@ -55,13 +55,15 @@ def _lib():
         lib.kv_evict_plan_set_debug.argtypes = [vp, ctypes.c_uint64, i32]
         lib.kv_evict_score.argtypes = [vp] * 7
         lib.kv_evict_select.argtypes = [vp] * 11
+        lib.kv_evict_select_noalloc.argtypes = [vp] * 10
         lib.kv_evict_gather.argtypes = [vp] * 7
         lib.kv_evict_status.argtypes = [vp, vp, vp]
         lib.kv_evict_profile.argtypes = [i32, vp, i32, vp, vp]
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
         lib.kv_evict_strerror.restype = ctypes.c_char_p
         for name in ("kv_evict_plan", "kv_evict_plan_set_debug", "kv_evict_score", "kv_evict_select",
-                     "kv_evict_gather", "kv_evict_status", "kv_evict_profile"):
+                     "kv_evict_select_noalloc", "kv_evict_gather", "kv_evict_status",
+                     "kv_evict_profile"):
             getattr(lib, name).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -148,6 +150,19 @@ class Plan:
                                       l1.ctypes.data, l2.ctypes.data, _ptr(indices), _ptr(order),
                                       _ptr(margins), _ptr(ws), _stream_ptr(stream)),
                "kv_evict_select")
+
+    def select_noalloc(self, mu, sigma, k, lambda1, lambda2, indices, order=None, margins=None,
+                       stream=None):
+        """kv_evict_select without a workspace, for callers that cannot allocate
+        device memory while they evict; its scratch is a fixed 16 MiB array inside
+        the library (at most N_L * Hkv * SL = 4194304 tokens per call)."""
+        l1 = np.ascontiguousarray(lambda1, dtype=np.float32)
+        l2 = np.ascontiguousarray(lambda2, dtype=np.float32)
+        assert l1.shape == (self.spec["num_layers"],) and l2.shape == l1.shape
+        _check(_lib().kv_evict_select_noalloc(self._h, _ptr(mu), _ptr(sigma), _ptr(k),
+                                              l1.ctypes.data, l2.ctypes.data, _ptr(indices),
+                                              _ptr(order), _ptr(margins), _stream_ptr(stream)),
+               "kv_evict_select_noalloc")
 
     def gather(self, k, v, indices, k_out, v_out, stream=None):
         _check(_lib().kv_evict_gather(self._h, _ptr(k), _ptr(v), _ptr(indices), _ptr(k_out),
