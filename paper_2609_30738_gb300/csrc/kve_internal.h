@@ -13,7 +13,7 @@ namespace kve {
 
 constexpr int kHeadDim = 128;      // d supported by this build
 constexpr int kTileKeys = 128;     // keys per MMA tile (one TMEM accumulator)
-constexpr int kSplitTiles = 4;     // tiles per work item
+constexpr int kSplitTiles = 8;     // tiles per work item
 constexpr int kSplitKeys = kTileKeys * kSplitTiles;
 constexpr int kMaxRows = 128;      // n = G*W window rows per unit, padded to one M tile
 constexpr int kMaxReq = 64;        // requests per call

@@ -4,15 +4,15 @@
 // L prefix keys through a causal softmax; mu_i and sigma_i are the mean and the
 // sample standard deviation of A[., i] over the n rows.
 //
-// Work is cut into items of up to 512 keys (4 tiles of 128). Each item runs in one
-// of two phases on a persistent, warp-specialised CTA:
+// Work is cut into items of up to kSplitKeys keys (tiles of 128). Each item runs in
+// one of two phases on a persistent, warp-specialised CTA:
 //   phase 0 (row statistics):   D[row][key] = Q K^T on tcgen05 (rows on TMEM lanes);
 //                               each epilogue thread owns one row and keeps the
 //                               running max m and sum Z = sum 2^(alpha*l - m) of its
-//                               row over the item's keys, then publishes (m, Z).
-//                               The last item of a unit to publish merges all of
-//                               them into beta_r = log2 of the row's softmax
-//                               normaliser and raises the unit's ready flag.
+//                               row; the item's (m, Z) per row are published, and
+//                               the last item of a unit to publish merges them into
+//                               beta_r = log2 of the row's softmax normaliser and
+//                               raises the unit's ready flag.
 //   phase 1 (column statistics): D[key][row] = K Q^T (keys on TMEM lanes); each
 //                               epilogue thread owns one key, forms
 //                               A = 2^(alpha*l - beta_r) for its n rows and reduces
@@ -21,17 +21,28 @@
 // before any phase-1 item of it, and phase-1 items trail phase-0 items by `lag`
 // items so that their K tiles are still in L2. A CTA processes its claims in
 // order, so a phase-1 item only ever waits for phase-0 items claimed before it;
-// the wait is bounded and reports KVE_ETIMEOUT instead of hanging.
+// every wait is bounded and a timeout is reported as KVE_ETIMEOUT.
 //
-// Roles: warp 0 claims items and issues TMA loads, warp 1 owns TMEM and issues
-// the MMAs, warps 2-5 run the epilogue (warp w reads TMEM lanes 32*(w%4)..+31).
+// Roles: warp 0 claims items and issues TMA loads; warp 1 owns TMEM and issues the
+// MMAs; warp 2 (sync) does all cross-CTA work in claim order -- it publishes the
+// row statistics of phase-0 items, merges a unit's statistics when its last item
+// arrives, and stages -beta of phase-1 items in shared memory ahead of use; warps
+// 3-10 run the epilogue in two groups of four (warp w reads TMEM lanes
+// 32*(w%4)..+31), the groups taking alternate tiles. The epilogue warps never
+// touch global synchronisation; they only compute, write shared memory and
+// arrive on mbarriers.
+#include <cstddef>
+
 #include "kve_internal.h"
 #include "kve_ptx.cuh"
 
 namespace kve {
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 352;
+constexpr int kSyncWarp = 2;
+constexpr int kEpiWarp0 = 3;
+constexpr int kEpiWarps = 8;
 constexpr int kQBufs = 2;
 constexpr int kKStages = 4;
 constexpr int kAccBufs = 4;      // 4 x 128 TMEM columns
@@ -47,14 +58,17 @@ struct ScoreCtl {
   uint64_t k_full[kKStages], k_empty[kKStages];
   uint64_t acc_full[kAccBufs], acc_empty[kAccBufs];
   uint64_t item_full[kItemSlots], item_empty[kItemSlots];
-  uint64_t epi_bar;
+  uint64_t pub_full[kItemSlots];    // epilogue -> sync warp, once per item
+  uint64_t beta_full[kItemSlots];   // sync warp -> epilogue, once per item
   int64_t item_ring[kItemSlots];
   uint32_t tmem_base;
   volatile int abort;
-  volatile int is_last;
-  float nbeta[kMaxRows];
-  int32_t roww[kMaxRows];
+  int32_t roww[kMaxRows];                            // r % W
+  alignas(16) float2 comb[kItemSlots][2][kMaxRows];  // per group (m, Z) of a row item
+  alignas(16) float nbeta[kItemSlots][kMaxRows];     // -beta of a column item
 };
+static_assert(offsetof(ScoreCtl, nbeta) % 16 == 0, "nbeta is read with 16-byte loads");
+static_assert(offsetof(ScoreCtl, comb) % 16 == 0, "comb holds float2");
 
 struct Claim {
   int phase;
@@ -99,32 +113,34 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64
   return __all_sync(0xffffffffu, ok);
 }
 
-// Bounded barrier among the 4 epilogue warps (an mbarrier with 4 arrivals).
-__device__ __forceinline__ bool epi_sync(ScoreCtl& ctl, uint32_t& phase, uint64_t limit) {
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) mbar_arrive(&ctl.epi_bar);
-  const bool ok = warp_wait(&ctl.epi_bar, phase, limit, &ctl.abort);
-  phase ^= 1u;
-  return ok;
+// Merge of two (m, Z) pairs in log2 units: Z counts 2^(x - m).
+__device__ __forceinline__ float2 merge_mz(float2 a, float2 b) {
+  const float m = fmaxf(a.x, b.x);
+  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
+  float z = 0.f;
+  if (a.x != -INFINITY) z = fmaf(a.y, ex2(a.x - m), z);
+  if (b.x != -INFINITY) z = fmaf(b.y, ex2(b.x - m), z);
+  return make_float2(m, z);
 }
 
 // ---------------------------------------------------------------- epilogue, phase 0
 
 template <bool kFull>
 __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, int split, int64_t p,
-                                              uint32_t& ai, uint32_t& epi_phase) {
+                                              const UnitInfo& u, int split, uint32_t slot,
+                                              uint32_t& ai) {
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
+  const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;   // 0 or 1
   const int row = quad * 32 + lane;
-  const int n = P.g.n_rows;
   const int W = P.g.window;
   const int lim_all = u.L - W;                 // keys <= lim_all are seen by every row
   const int lim = u.L - W + ctl.roww[row];     // last key this row sees
   const int ntiles = item_tiles(u.L, split);
   const float alpha = P.alpha;
   float m = -INFINITY, Z = 0.f;
-  for (int t = 0; t < ntiles; ++t) {
+  for (int t = 0; t < ntiles; ++t, ++ai) {
+    if (static_cast<int>(ai & 1u) != grp) continue;   // the other group's tile
     const uint32_t ab = ai % kAccBufs;
     if (!warp_wait(&ctl.acc_full[ab], (ai / kAccBufs) & 1u, P.wait_limit_ns, &ctl.abort))
       return false;
@@ -137,7 +153,6 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
-    ++ai;
     const int key0 = split * kSplitKeys + t * kTileKeys;
     if (key0 + kTileKeys - 1 > lim_all) {
 #pragma unroll
@@ -150,50 +165,26 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
     mx = fmaxf(mx, v[127]);
     const float mn = fmaxf(m, mx * alpha);
     if (mn != -INFINITY) {
-      float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+      const float2 a2 = make_float2(alpha, alpha);
+      const float2 nm2 = make_float2(-mn, -mn);
+      float2 s0 = make_float2(0.f, 0.f), s1 = s0, s2 = s0, s3 = s0;
 #pragma unroll
-      for (int j = 0; j < 128; j += 4) {
-        s0 += ex2(fmaf(v[j + 0], alpha, -mn));
-        s1 += ex2(fmaf(v[j + 1], alpha, -mn));
-        s2 += ex2(fmaf(v[j + 2], alpha, -mn));
-        s3 += ex2(fmaf(v[j + 3], alpha, -mn));
+      for (int j = 0; j < 128; j += 8) {
+        float2 x[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) x[k] = ffma2(make_float2(v[j + 2 * k], v[j + 2 * k + 1]), a2, nm2);
+        s0 = fadd2(s0, make_float2(ex2(x[0].x), ex2(x[0].y)));
+        s1 = fadd2(s1, make_float2(ex2(x[1].x), ex2(x[1].y)));
+        s2 = fadd2(s2, make_float2(ex2(x[2].x), ex2(x[2].y)));
+        s3 = fadd2(s3, make_float2(ex2(x[3].x), ex2(x[3].y)));
       }
+      const float2 ss = fadd2(fadd2(s0, s1), fadd2(s2, s3));
       const float scale = (m == -INFINITY) ? 0.f : ex2(m - mn);
-      Z = fmaf(Z, scale, (s0 + s1) + (s2 + s3));
+      Z = fmaf(Z, scale, ss.x + ss.y);
       m = mn;
     }
   }
-  if (kFull || row < n) {
-    P.partial[p * kMaxRows + row] = make_float2(m, Z);
-  }
-  __threadfence();
-  if (!epi_sync(ctl, epi_phase, P.wait_limit_ns)) return false;
-  if (threadIdx.x == 64) {
-    int last = 0;
-    if (!(P.fault == 1 && u.unit == 0)) {
-      const uint32_t old = atomicAdd(&P.counts[u.unit], 1u);
-      last = (old == static_cast<uint32_t>(u.splits - 1));
-    }
-    ctl.is_last = last;
-  }
-  if (!epi_sync(ctl, epi_phase, P.wait_limit_ns)) return false;
-  if (ctl.is_last) {
-    __threadfence();
-    if (kFull || row < n) {
-      float mg = -INFINITY;
-      for (int s = 0; s < u.splits; ++s)
-        mg = fmaxf(mg, __ldcg(&P.partial[(u.item0 + s) * kMaxRows + row]).x);
-      float zg = 0.f;
-      for (int s = 0; s < u.splits; ++s) {
-        const float2 pz = __ldcg(&P.partial[(u.item0 + s) * kMaxRows + row]);
-        if (pz.x != -INFINITY) zg = fmaf(pz.y, ex2(pz.x - mg), zg);
-      }
-      __stcg(&P.beta[u.unit * kMaxRows + row], mg + lg2(zg));
-    }
-    __threadfence();
-    if (!epi_sync(ctl, epi_phase, P.wait_limit_ns)) return false;
-    if (threadIdx.x == 64) st_release_gpu(&P.flags[u.unit], 1u);
-  }
+  ctl.comb[slot][grp][row] = make_float2(m, Z);
   return true;
 }
 
@@ -201,38 +192,23 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
 
 template <bool kFull>
 __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, int split, uint32_t& ai,
-                                              uint32_t& epi_phase) {
+                                              const UnitInfo& u, int split, uint32_t slot,
+                                              uint32_t& ai) {
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
+  const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;
   const int tl = quad * 32 + lane;         // key within the tile
   const int n = kFull ? kMaxRows : P.g.n_rows;
   const int nch = kFull ? 4 : (n + 31) / 32;
   const int W = P.g.window;
   const float alpha = P.alpha;
-  // wait for the unit's merged row statistics
-  if (threadIdx.x == 64) {
-    const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
-    const volatile uint32_t* errw = P.err;
-    uint32_t ns = 32;
-    while (ld_acquire_gpu(&P.flags[u.unit]) == 0u) {
-      if (*errw != 0u || global_timer_ns() > deadline) {
-        set_error(P, ctl, 1u);
-        break;
-      }
-      __nanosleep(ns);
-      if (ns < 1024) ns *= 2;
-    }
-  }
-  if (!epi_sync(ctl, epi_phase, P.wait_limit_ns)) return false;
-  if (ctl.abort) return false;
-  ctl.nbeta[tl] = (tl < P.g.n_rows) ? -__ldcg(&P.beta[u.unit * kMaxRows + tl]) : -INFINITY;
-  if (!epi_sync(ctl, epi_phase, P.wait_limit_ns)) return false;
-
   const int ntiles = item_tiles(u.L, split);
   const float inv_n = 1.0f / static_cast<float>(n);
   const float inv_n1 = n > 1 ? 1.0f / static_cast<float>(n - 1) : 0.f;
-  for (int t = 0; t < ntiles; ++t) {
+  const float4* nb4 = reinterpret_cast<const float4*>(ctl.nbeta[slot]);
+  const float2 a2 = make_float2(alpha, alpha);
+  for (int t = 0; t < ntiles; ++t, ++ai) {
+    if (static_cast<int>(ai & 1u) != grp) continue;
     const uint32_t ab = ai % kAccBufs;
     if (!warp_wait(&ctl.acc_full[ab], (ai / kAccBufs) & 1u, P.wait_limit_ns, &ctl.abort))
       return false;
@@ -246,12 +222,19 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
-    ++ai;
     const int key = split * kSplitKeys + t * kTileKeys + tl;
     // A[r] = 2^(alpha*l - beta_r); rows that do not see this key (causal) get 0
 #pragma unroll
-    for (int r = 0; r < 128; ++r) {
-      if (kFull || r < n) v[r] = ex2(fmaf(v[r], alpha, ctl.nbeta[r]));
+    for (int r = 0; r < 128; r += 4) {
+      if (kFull || r < n) {
+        const float4 b = nb4[r >> 2];
+        const float2 x0 = ffma2(make_float2(v[r], v[r + 1]), a2, make_float2(b.x, b.y));
+        const float2 x1 = ffma2(make_float2(v[r + 2], v[r + 3]), a2, make_float2(b.z, b.w));
+        v[r] = ex2(x0.x);
+        v[r + 1] = ex2(x0.y);
+        v[r + 2] = ex2(x1.x);
+        v[r + 3] = ex2(x1.y);
+      }
     }
     if (key > u.L - W) {
       const int rel = key - (u.L - W);
@@ -259,30 +242,140 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
       for (int r = 0; r < 128; ++r)
         if ((kFull || r < n) && rel > ctl.roww[r]) v[r] = 0.f;
     }
-    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    float mu, sigma;
+    if (kFull) {
+      float2 a0 = make_float2(0.f, 0.f), a1 = a0, a2s = a0, a3 = a0;
 #pragma unroll
-    for (int r = 0; r < 128; r += 4) {
-      if (kFull || r + 0 < n) a0 += v[r + 0];
-      if (kFull || r + 1 < n) a1 += v[r + 1];
-      if (kFull || r + 2 < n) a2 += v[r + 2];
-      if (kFull || r + 3 < n) a3 += v[r + 3];
-    }
-    const float mu = ((a0 + a1) + (a2 + a3)) * inv_n;
-    float q0 = 0.f, q1 = 0.f, q2 = 0.f, q3 = 0.f;
+      for (int r = 0; r < 128; r += 8) {
+        a0 = fadd2(a0, make_float2(v[r], v[r + 1]));
+        a1 = fadd2(a1, make_float2(v[r + 2], v[r + 3]));
+        a2s = fadd2(a2s, make_float2(v[r + 4], v[r + 5]));
+        a3 = fadd2(a3, make_float2(v[r + 6], v[r + 7]));
+      }
+      const float2 as = fadd2(fadd2(a0, a1), fadd2(a2s, a3));
+      mu = (as.x + as.y) * inv_n;
+      const float2 nmu = make_float2(-mu, -mu);
+      float2 q0 = make_float2(0.f, 0.f), q1 = q0, q2 = q0, q3 = q0;
 #pragma unroll
-    for (int r = 0; r < 128; r += 4) {
-      float d;
-      if (kFull || r + 0 < n) { d = v[r + 0] - mu; q0 = fmaf(d, d, q0); }
-      if (kFull || r + 1 < n) { d = v[r + 1] - mu; q1 = fmaf(d, d, q1); }
-      if (kFull || r + 2 < n) { d = v[r + 2] - mu; q2 = fmaf(d, d, q2); }
-      if (kFull || r + 3 < n) { d = v[r + 3] - mu; q3 = fmaf(d, d, q3); }
+      for (int r = 0; r < 128; r += 8) {
+        const float2 d0 = fadd2(make_float2(v[r], v[r + 1]), nmu);
+        const float2 d1 = fadd2(make_float2(v[r + 2], v[r + 3]), nmu);
+        const float2 d2 = fadd2(make_float2(v[r + 4], v[r + 5]), nmu);
+        const float2 d3 = fadd2(make_float2(v[r + 6], v[r + 7]), nmu);
+        q0 = ffma2(d0, d0, q0);
+        q1 = ffma2(d1, d1, q1);
+        q2 = ffma2(d2, d2, q2);
+        q3 = ffma2(d3, d3, q3);
+      }
+      const float2 qs = fadd2(fadd2(q0, q1), fadd2(q2, q3));
+      sigma = sqrtf((qs.x + qs.y) * inv_n1);
+    } else {
+      float a = 0.f;
+#pragma unroll
+      for (int r = 0; r < 128; ++r)
+        if (r < n) a += v[r];
+      mu = a * inv_n;
+      float q = 0.f;
+#pragma unroll
+      for (int r = 0; r < 128; ++r)
+        if (r < n) {
+          const float d = v[r] - mu;
+          q = fmaf(d, d, q);
+        }
+      sigma = sqrtf(q * inv_n1);
     }
-    const float sigma = sqrtf(((q0 + q1) + (q2 + q3)) * inv_n1);
     if (key < u.L) {
       __stcs(&P.mu[u.mu_off + key], mu);
       __stcs(&P.sigma[u.mu_off + key], sigma);
     }
   }
+  return true;
+}
+
+// ---------------------------------------------------------------- sync warp
+
+// Phase-0 item: merge the two groups' (m, Z) per row, publish them, count the item,
+// and if it is the unit's last, merge all of the unit's items into beta.
+__device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ctl,
+                                              const UnitInfo& u, int64_t p, uint32_t slot) {
+  const int lane = threadIdx.x & 31;
+  const int n = P.g.n_rows;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int row = lane + 32 * k;
+    const float2 mz = merge_mz(ctl.comb[slot][0][row], ctl.comb[slot][1][row]);
+    if (row < n) P.partial[p * kMaxRows + row] = mz;
+  }
+  __threadfence();
+  __syncwarp();
+  int last = 0;
+  if (lane == 0 && !(P.fault == 1 && u.unit == 0)) {
+    const uint32_t old = atomicAdd(&P.counts[u.unit], 1u);
+    last = (old == static_cast<uint32_t>(u.splits - 1));
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (last) {
+    __threadfence();
+    float2 acc[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) acc[k] = make_float2(-INFINITY, 0.f);
+    for (int s0 = 0; s0 < u.splits; s0 += 16) {
+      float2 pz[4][16];
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int row = lane + 32 * k;
+          pz[k][j] = (s0 + j < u.splits && row < n)
+                         ? __ldcg(&P.partial[(u.item0 + s0 + j) * kMaxRows + row])
+                         : make_float2(-INFINITY, 0.f);
+        }
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j < 16; ++j) acc[k] = merge_mz(acc[k], pz[k][j]);
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int row = lane + 32 * k;
+      if (row < n) __stcg(&P.beta[u.unit * kMaxRows + row], acc[k].x + lg2(acc[k].y));
+    }
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) st_release_gpu(&P.flags[u.unit], 1u);
+  }
+  return true;
+}
+
+// Phase-1 item: wait for the unit's merged statistics and stage -beta.
+__device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ctl,
+                                              const UnitInfo& u, uint32_t slot) {
+  const int lane = threadIdx.x & 31;
+  int ok = 1;
+  if (lane == 0) {
+    const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
+    const volatile uint32_t* errw = P.err;
+    uint32_t ns = 32;
+    while (ld_acquire_gpu(&P.flags[u.unit]) == 0u) {
+      if (*errw != 0u || ctl.abort || global_timer_ns() > deadline) {
+        ok = 0;
+        break;
+      }
+      __nanosleep(ns);
+      if (ns < 512) ns *= 2;
+    }
+  }
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (!ok) return false;
+  __syncwarp();   // orders every lane's loads after lane 0's acquire
+  const int n = P.g.n_rows;
+  float4 b;
+  const int r0 = 4 * lane;
+  b.x = r0 + 0 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 0]) : -INFINITY;
+  b.y = r0 + 1 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 1]) : -INFINITY;
+  b.z = r0 + 2 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 2]) : -INFINITY;
+  b.w = r0 + 3 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 3]) : -INFINITY;
+  reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
   return true;
 }
 
@@ -308,10 +401,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int i = 0; i < kQBufs; ++i) { mbar_init(&ctl.q_full[i], 1); mbar_init(&ctl.q_empty[i], 1); }
     for (int i = 0; i < kKStages; ++i) { mbar_init(&ctl.k_full[i], 1); mbar_init(&ctl.k_empty[i], 1); }
     for (int i = 0; i < kAccBufs; ++i) { mbar_init(&ctl.acc_full[i], 1); mbar_init(&ctl.acc_empty[i], 4); }
-    for (int i = 0; i < kItemSlots; ++i) { mbar_init(&ctl.item_full[i], 1); mbar_init(&ctl.item_empty[i], 5); }
-    mbar_init(&ctl.epi_bar, 4);
+    for (int i = 0; i < kItemSlots; ++i) {
+      mbar_init(&ctl.item_full[i], 1);
+      mbar_init(&ctl.item_empty[i], 2 + kEpiWarps);   // MMA + sync + epilogue warps
+      mbar_init(&ctl.pub_full[i], kEpiWarps);
+      mbar_init(&ctl.beta_full[i], 1);
+    }
     ctl.abort = 0;
-    ctl.is_last = 0;
     fence_mbar_init();
     prefetch_tensormap(&tm_q);
     prefetch_tensormap(&tm_k);
@@ -334,9 +430,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_keep = l2_policy_evict_last();
       const uint64_t pol_drop = l2_policy_evict_first();
       bool ok = true;
+      // the next claim is requested one item ahead so that its round trip overlaps
+      // the loads of the current item (claims are still processed in order)
+      uint32_t next = atomicAdd(P.claim, 1u);
       for (;;) {
-        int64_t c = ctl.abort ? total_claims : static_cast<int64_t>(atomicAdd(P.claim, 1u));
+        int64_t c = ctl.abort ? total_claims : static_cast<int64_t>(next);
         if (c > total_claims) c = total_claims;
+        if (c < total_claims) next = atomicAdd(P.claim, 1u);
         const uint32_t slot = it % kItemSlots;
         if (!mbar_wait(&ctl.item_empty[slot], ((it / kItemSlots) & 1u) ^ 1u,
                        global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
@@ -460,30 +560,71 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (issued)
         mbar_wait(&ctl.acc_full[last_ab], last_par, global_timer_ns() + P.wait_limit_ns, &no_abort);
     }
-  } else {
-    // ------------------------------------------------------------ epilogue
-    uint32_t it = 0, ai = 0, epi_phase = 0;
+  } else if (warp == kSyncWarp) {
+    // ------------------------------------------------------------ sync warp
+    uint32_t it = 0;
     for (;;) {
       const uint32_t slot = it % kItemSlots;
-      if (!warp_wait(&ctl.item_full[slot], (it / kItemSlots) & 1u, P.wait_limit_ns, &ctl.abort)) {
+      const uint32_t par = (it / kItemSlots) & 1u;
+      if (!warp_wait(&ctl.item_full[slot], par, P.wait_limit_ns, &ctl.abort)) {
         set_error(P, ctl, 1u);
         break;
       }
       const int64_t c = ctl.item_ring[slot];
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
-      ++it;
       if (c < 0) break;
       const Claim cl = decode_claim(c, n1, P.lag);
       int split;
       const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
-      const bool ok = (cl.phase == 0)
-                          ? rowstats_item<kFull>(P, ctl, u, split, cl.p, ai, epi_phase)
-                          : colstats_item<kFull>(P, ctl, u, split, ai, epi_phase);
+      bool ok;
+      if (cl.phase == 0) {
+        if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);      // nothing to stage
+        ok = warp_wait(&ctl.pub_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
+             sync_rowstats(P, ctl, u, cl.p, slot);
+      } else {
+        ok = sync_colstats(P, ctl, u, slot);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);
+      }
       if (!ok) {
         set_error(P, ctl, 1u);
         break;
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
+      ++it;
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    uint32_t it = 0, ai = 0;
+    for (;;) {
+      const uint32_t slot = it % kItemSlots;
+      const uint32_t par = (it / kItemSlots) & 1u;
+      if (!warp_wait(&ctl.item_full[slot], par, P.wait_limit_ns, &ctl.abort)) {
+        set_error(P, ctl, 1u);
+        break;
+      }
+      const int64_t c = ctl.item_ring[slot];
+      if (c < 0) break;
+      const Claim cl = decode_claim(c, n1, P.lag);
+      int split;
+      const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
+      bool ok;
+      if (cl.phase == 0) {
+        ok = rowstats_item<kFull>(P, ctl, u, split, slot, ai);
+      } else {
+        ok = warp_wait(&ctl.beta_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
+             colstats_item<kFull>(P, ctl, u, split, slot, ai);
+      }
+      if (!ok) {
+        set_error(P, ctl, 1u);
+        break;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&ctl.pub_full[slot]);
+        mbar_arrive(&ctl.item_empty[slot]);
+      }
+      ++it;
     }
   }
 
