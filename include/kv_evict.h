@@ -75,8 +75,8 @@ typedef struct {
   int32_t window;           /* W >= 1, with G*W <= 128                         */
   int32_t budget;           /* B >= 1 kept candidates per unit (the window is
                                kept in addition)                               */
-  int32_t pool_kernel;      /* odd k >= 1; max-pool of mu and sigma, stride 1,
-                               window clipped to [0, Lc); 1 = no pooling       */
+  int32_t pool_kernel;      /* odd k, 1 <= k <= 255; max-pool of mu and sigma,
+                               stride 1, window clipped to [0, Lc); 1 = none    */
   int32_t candidate_factor; /* greedy pool C = min(factor*B, Lc); Section 3.2
                                uses 4; 0 = every candidate                     */
   float norm_eps;           /* positive clamp of max_j s_j in Eq. 5            */

@@ -74,7 +74,8 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   if (c.head_dim != kHeadDim) return KVE_EINVAL;
   const int G = c.num_q_heads / c.num_kv_heads;
   if (c.window < 1 || static_cast<int64_t>(G) * c.window > kMaxRows) return KVE_EINVAL;
-  if (c.budget < 1 || c.pool_kernel < 1 || c.pool_kernel % 2 == 0) return KVE_EINVAL;
+  if (c.budget < 1 || c.pool_kernel < 1 || c.pool_kernel > 255 || c.pool_kernel % 2 == 0)
+    return KVE_EINVAL;
   if (c.candidate_factor < 0 || !(c.norm_eps > 0.f) || !std::isfinite(c.norm_eps)) return KVE_EINVAL;
   if (n_req < 1 || n_req > kMaxReq) return KVE_EINVAL;
 

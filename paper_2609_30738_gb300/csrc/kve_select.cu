@@ -5,8 +5,8 @@
 //     and form the base score s_i = mu_i + lambda1 sigma_i (Eq. 2 without corr);
 //     s is stored as an order-preserving 32-bit key in the workspace;
 //  2. find the C = min(factor*B, Lc) largest keys (Section 3.2: the greedy runs on
-//     the top 4B tokens) by an MSB-first radix select; ties at the cut go to the
-//     lower positions;
+//     the top 4B tokens) by an MSB-first radix select with 12/12/8-bit digits;
+//     ties at the cut go to the lower positions;
 //  3. normalise s~ = s / max(max s, eps) (Eq. 5) and stage the candidate keys
 //     (bf16) and their inverse norms in shared memory, candidates sorted by
 //     position so that "lower slot" means "lower position";
@@ -16,6 +16,7 @@
 //     both corr(i, {}) and the clamp at 0);
 //  5. write the admitted positions ascending (and optionally in admission order,
 //     with the best-minus-second margin of every admission).
+// The block has one thread per pool slot (256 for C <= 256, else 512).
 #include <mutex>
 
 #include "kve_internal.h"
@@ -23,9 +24,13 @@
 namespace kve {
 namespace {
 
-constexpr int kSelThreads = 512;
-constexpr int kMaxCand = 512;
 constexpr int kChunks = kHeadDim / 8;   // 16-byte chunks of a key row
+constexpr int kBins = 4096;             // radix digits of the first two passes
+constexpr int kPoolRun = 7;             // consecutive pooled outputs per run (odd: the
+                                        // runs of a warp start on distinct banks)
+constexpr int kPoolRuns = 4;            // runs per thread and tile
+constexpr int kBatch = 16;              // key loads in flight per thread
+constexpr int kTieCap = 2048;           // cut ties gathered in shared memory
 
 __device__ __forceinline__ uint32_t ord_key(float f) {
   const uint32_t u = __float_as_uint(f + 0.0f);   // -0 -> +0
@@ -37,33 +42,25 @@ __device__ __forceinline__ float unord_key(uint32_t k) {
   return __uint_as_float(u);
 }
 
-struct SelShared {
-  uint32_t hist[256];
-  uint32_t warp_tot[kSelThreads / 32];
-  unsigned long long red[2][kSelThreads / 32][2];
-  uint32_t prefix, need, cnt, maxkey, taken_tot;
+template <int NT>
+struct SelSmall {
+  uint32_t warp_tot[NT / 32];
+  uint32_t red[2][NT / 32][4];   // per warp: best key, best slot, second key
+  uint32_t prefix, need, cnt, maxkey, teq;
 };
 
-// top-2 of two top-2 lists (keys unique except zeros)
-__device__ __forceinline__ void top2_merge(unsigned long long& b1, unsigned long long& b2,
-                                           unsigned long long o1, unsigned long long o2) {
-  const unsigned long long hi = b1 > o1 ? b1 : o1;
-  const unsigned long long lo = b1 > o1 ? o1 : b1;
-  const unsigned long long sec = b2 > o2 ? b2 : o2;
-  b1 = hi;
-  b2 = lo > sec ? lo : sec;
-}
-
-// Exclusive prefix count of `flag` over the block in thread order; returns the
-// prefix and writes the block total to *total (all threads).
-__device__ __forceinline__ uint32_t block_excl_count(bool flag, SelShared& sh, uint32_t* total) {
+// Exclusive prefix count of `flag` over the block in thread order; the block
+// total is returned in *total (all threads).
+template <int NT>
+__device__ __forceinline__ uint32_t block_excl_count(bool flag, SelSmall<NT>& sh, uint32_t* total) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t bal = __ballot_sync(0xffffffffu, flag);
   const uint32_t in_warp = __popc(bal & ((1u << lane) - 1u));
   if (lane == 0) sh.warp_tot[warp] = __popc(bal);
   __syncthreads();
   uint32_t before = 0, tot = 0;
-  for (int w = 0; w < kSelThreads / 32; ++w) {
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) {
     const uint32_t x = sh.warp_tot[w];
     if (w < warp) before += x;
     tot += x;
@@ -73,8 +70,29 @@ __device__ __forceinline__ uint32_t block_excl_count(bool flag, SelShared& sh, u
   return before + in_warp;
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_constant__ SelectParams P) {
-  __shared__ SelShared sh;
+// Exclusive suffix sum of `x` over the block (sum over higher thread indices).
+template <int NT>
+__device__ __forceinline__ uint32_t block_excl_suffix(uint32_t x, SelSmall<NT>& sh) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint32_t incl = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_down_sync(0xffffffffu, incl, o);
+    if (lane + o < 32) incl += y;
+  }
+  if (lane == 0) sh.warp_tot[warp] = incl;   // warp total
+  __syncthreads();
+  uint32_t after = 0;
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w)
+    if (w > warp) after += sh.warp_tot[w];
+  __syncthreads();
+  return incl - x + after;
+}
+
+template <int NT>
+__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams P) {
+  __shared__ SelSmall<NT> sh;
   extern __shared__ __align__(16) uint8_t dyn[];
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -92,22 +110,98 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   uint32_t* keys = P.keys + u.mu_off;
   const int h = P.pool_kernel / 2;
 
-  // shared arrays sized by the largest pool
-  uint4* kch = reinterpret_cast<uint4*>(dyn);                         // [kChunks][C]
-  int32_t* spos = reinterpret_cast<int32_t*>(kch + kChunks * kMaxCand); // [C] sorted positions
-  int32_t* cpos = spos + kMaxCand;                                     // [C] collected positions
-  float* st = reinterpret_cast<float*>(cpos + kMaxCand);               // [C] s~
-  float* inv = st + kMaxCand;                                          // [C] 1/|k|
+  // shared memory: [ big | spos | cpos | st | inv ]; `big` holds in turn the pooling
+  // tiles, the radix histogram and the staged candidate keys
+  uint8_t* big = dyn;
+  uint4* krow = reinterpret_cast<uint4*>(big);                                  // [NT][kChunks]
+  uint32_t* hist12 = reinterpret_cast<uint32_t*>(big);                          // [kBins] later passes
+  float* tmu = reinterpret_cast<float*>(big);                                   // pooling tiles
+  int32_t* spos = reinterpret_cast<int32_t*>(big + kChunks * NT * sizeof(uint4));
+  int32_t* cpos = spos + NT;
+  float* st = reinterpret_cast<float*>(cpos + NT);
+  float* inv = st + NT;
+  uint32_t* hist0 = reinterpret_cast<uint32_t*>(inv + NT);                      // [kBins] first pass
 
-  // 1. pooled base score as ordered keys
-  for (int i = tid; i < Lc; i += kSelThreads) {
-    const int lo = max(0, i - h), hi = min(Lc - 1, i + h);
-    float mh = mu[lo], sh_ = sg[lo];
-    for (int j = lo + 1; j <= hi; ++j) {
-      mh = fmaxf(mh, mu[j]);
-      sh_ = fmaxf(sh_, sg[j]);
+  for (int b = tid; b < kBins; b += NT) hist0[b] = 0;
+  __syncthreads();
+  // 1. pooled base score as ordered keys (and the histogram of their top 12 bits);
+  //    a tile holds kPoolRuns runs of kPoolRun
+  //    consecutive outputs per thread (run q of thread t starts at (q*NT + t)*kPoolRun)
+  {
+    constexpr int kTile = NT * kPoolRun * kPoolRuns;
+    const int tile_in = kTile + 2 * h;
+    float* tsg = tmu + tile_in;
+    for (int base = 0; base < Lc; base += kTile) {
+      {
+        // every load of the tile is issued before the first store (one round trip)
+        constexpr int kPer = (kTile + 2 * 127 + NT - 1) / NT;
+        float lm[kPer], ls[kPer];
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+          const int j = q * NT + tid;
+          const int i = base - h + j;
+          const bool in = (j < tile_in) && (i >= 0) && (i < Lc);
+          lm[q] = in ? __ldg(mu + i) : -INFINITY;
+          ls[q] = in ? __ldg(sg + i) : -INFINITY;
+        }
+#pragma unroll
+        for (int q = 0; q < kPer; ++q) {
+          const int j = q * NT + tid;
+          if (j < tile_in) {
+            tmu[j] = lm[q];
+            tsg[j] = ls[q];
+          }
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < kPoolRuns; ++q) {
+        const int o0 = (q * NT + tid) * kPoolRun;
+        if (h <= 3) {
+          // a 13-value window in registers covers the 7 outputs of the run for any
+          // kernel up to 7; out[r] = max of x[o0+r .. o0+r+2h] (tile coordinates)
+          float wm[kPoolRun + 6], ws[kPoolRun + 6];
+#pragma unroll
+          for (int j = 0; j < kPoolRun + 6; ++j) {
+            const bool in = j < kPoolRun + 2 * h;
+            wm[j] = in ? tmu[o0 + j] : -INFINITY;
+            ws[j] = in ? tsg[o0 + j] : -INFINITY;
+          }
+#pragma unroll
+          for (int r = 0; r < kPoolRun; ++r) {
+            float mh = wm[r], shh = ws[r];
+#pragma unroll
+            for (int j = 1; j <= 6; ++j)
+              if (j <= 2 * h) {
+                mh = fmaxf(mh, wm[r + j]);
+                shh = fmaxf(shh, ws[r + j]);
+              }
+            const int i = base + o0 + r;
+            if (i < Lc) {
+              const uint32_t k = ord_key(fmaf(lambda1, shh, mh));
+              keys[i] = k;
+              atomicAdd(&hist0[k >> 20], 1u);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int r = 0; r < kPoolRun; ++r) {
+            const int i = base + o0 + r;
+            if (i < Lc) {
+              float mh = tmu[o0 + r], shh = tsg[o0 + r];
+              for (int j = 1; j <= 2 * h; ++j) {
+                mh = fmaxf(mh, tmu[o0 + r + j]);
+                shh = fmaxf(shh, tsg[o0 + r + j]);
+              }
+              const uint32_t k = ord_key(fmaf(lambda1, shh, mh));
+              keys[i] = k;
+              atomicAdd(&hist0[k >> 20], 1u);
+            }
+          }
+        }
+      }
+      __syncthreads();
     }
-    keys[i] = ord_key(fmaf(lambda1, sh_, mh));
   }
   if (tid == 0) {
     sh.prefix = 0;
@@ -117,71 +211,105 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   }
   __syncthreads();
 
-  // 2. radix select of the C-th largest key
+  // 2. radix select of the C-th largest key: digits of 12, 12 and 8 bits
   uint32_t pmask = 0;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    if (tid < 256) sh.hist[tid] = 0;
+#pragma unroll 1
+  for (int pass = 0; pass < 3; ++pass) {
+    const int shift = pass == 0 ? 20 : (pass == 1 ? 8 : 0);
+    const int nb = pass == 2 ? 256 : kBins;
+    uint32_t* hist = pass == 0 ? hist0 : hist12;
+    if (pass > 0)
+      for (int b = tid; b < nb; b += NT) hist[b] = 0;
     __syncthreads();
     const uint32_t prefix = sh.prefix;
-    for (int i = tid; i < Lc; i += kSelThreads) {
-      const uint32_t k = __ldcg(&keys[i]);
-      if ((k & pmask) == prefix) atomicAdd(&sh.hist[(k >> shift) & 255u], 1u);
+    for (int i0 = 0; pass > 0 && i0 < Lc; i0 += NT * kBatch) {
+      uint32_t kb[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        kb[j] = i < Lc ? __ldcg(&keys[i]) : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        if ((i < Lc) && ((kb[j] & pmask) == prefix))
+          atomicAdd(&hist[(kb[j] >> shift) & static_cast<uint32_t>(nb - 1)], 1u);
+      }
     }
     __syncthreads();
-    if (warp == 0) {
-      // lane l owns bins 8l .. 8l+7; find the digit where the count from the top
-      // first reaches `need`
-      uint32_t c[8], s = 0;
-#pragma unroll
-      for (int b = 0; b < 8; ++b) { c[b] = sh.hist[8 * lane + b]; s += c[b]; }
-      // inclusive suffix sum over lanes >= lane, then exclusive (lanes > lane)
-      uint32_t incl = s;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t x = __shfl_down_sync(0xffffffffu, incl, o);
-        if (lane + o < 32) incl += x;
-      }
-      const uint32_t suffix = incl - s;
-      const uint32_t need = sh.need;
-      int found = -1;
-      uint32_t acc = suffix, above_digit = 0;
-      if (suffix < need && suffix + s >= need) {
-        for (int b = 7; b >= 0; --b) {
-          if (acc + c[b] >= need) { found = 8 * lane + b; above_digit = acc; break; }
-          acc += c[b];
+    // thread t owns bins [t*per, (t+1)*per); find the digit where the count from
+    // the top first reaches `need`
+    const int per = nb / NT > 0 ? nb / NT : 1;
+    const int b0 = tid * per;
+    uint32_t mine = 0;
+    if (b0 < nb)
+      for (int b = 0; b < per; ++b) mine += hist[b0 + b];
+    const uint32_t above = block_excl_suffix<NT>(mine, sh);
+    const uint32_t need = sh.need;
+    if (b0 < nb && above < need && above + mine >= need) {
+      uint32_t acc = above;
+      for (int b = per - 1; b >= 0; --b) {
+        const uint32_t c = hist[b0 + b];
+        if (acc + c >= need) {
+          sh.prefix = prefix | (static_cast<uint32_t>(b0 + b) << shift);
+          sh.need = need - acc;
+          break;
         }
-      }
-      const uint32_t bal = __ballot_sync(0xffffffffu, found >= 0);
-      const int src = __ffs(bal) - 1;
-      const int digit = __shfl_sync(0xffffffffu, found, src);
-      const uint32_t abv = __shfl_sync(0xffffffffu, above_digit, src);
-      if (lane == 0) {
-        sh.prefix = prefix | (static_cast<uint32_t>(digit) << shift);
-        sh.need = need - abv;
+        acc += c;
       }
     }
-    pmask |= 0xFFu << shift;
+    pmask |= static_cast<uint32_t>(nb - 1) << shift;
     __syncthreads();
   }
   const uint32_t T = sh.prefix;
   const uint32_t needT = sh.need;   // keys equal to T to take, lowest positions first
 
-  // 3a. every key above the threshold
-  for (int i = tid; i < Lc; i += kSelThreads) {
-    const uint32_t k = __ldcg(&keys[i]);
-    if (k > T) cpos[atomicAdd(&sh.cnt, 1u)] = i;
+  // 3. every key above the threshold, and the positions of the keys equal to it
+  if (tid == 0) sh.teq = 0;
+  __syncthreads();
+  int32_t* ties = reinterpret_cast<int32_t*>(big);   // [kTieCap], the histogram is dead
+  for (int i0 = 0; i0 < Lc; i0 += NT * kBatch) {
+    uint32_t kb[kBatch];
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int i = i0 + j * NT + tid;
+      kb[j] = i < Lc ? __ldcg(&keys[i]) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < kBatch; ++j) {
+      const int i = i0 + j * NT + tid;
+      if (i < Lc) {
+        if (kb[j] > T) {
+          cpos[atomicAdd(&sh.cnt, 1u)] = i;
+        } else if (kb[j] == T) {
+          const uint32_t e = atomicAdd(&sh.teq, 1u);
+          if (e < kTieCap) ties[e] = i;
+        }
+      }
+    }
   }
   __syncthreads();
   const uint32_t n_above = sh.cnt;
-  // 3b. the needT lowest positions whose key equals T
-  uint32_t taken = 0;
-  for (int base = 0; base < Lc && taken < needT; base += kSelThreads) {
-    const int i = base + tid;
-    const bool f = (i < Lc) && (__ldcg(&keys[i]) == T);
-    uint32_t tot;
-    const uint32_t pre = block_excl_count(f, sh, &tot);
-    if (f && taken + pre < needT) cpos[n_above + taken + pre] = i;
-    taken += tot;
+  const uint32_t n_eq = sh.teq;
+  if (n_eq <= kTieCap) {
+    // the needT lowest positions among the ties, by rank
+    for (uint32_t e = tid; e < n_eq; e += NT) {
+      const int pos = ties[e];
+      uint32_t rank = 0;
+      for (uint32_t f = 0; f < n_eq; ++f) rank += (ties[f] < pos);
+      if (rank < needT) cpos[n_above + rank] = pos;
+    }
+  } else {
+    // many equal keys: ordered block scan over the positions
+    uint32_t taken = 0;
+    for (int base = 0; base < Lc && taken < needT; base += NT) {
+      const int i = base + tid;
+      const bool f = (i < Lc) && (__ldcg(&keys[i]) == T);
+      uint32_t tot;
+      const uint32_t pre = block_excl_count<NT>(f, sh, &tot);
+      if (f && taken + pre < needT) cpos[n_above + taken + pre] = i;
+      taken += tot;
+    }
   }
   __syncthreads();
 
@@ -195,18 +323,26 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
   }
   __syncthreads();
   const float smax = fmaxf(unord_key(sh.maxkey), P.norm_eps);
-  float corr = 0.f;
-  bool mine_taken = tid >= C;
-  if (tid < C) {
-    const int pos = spos[tid];
-    st[tid] = __fdiv_rn(unord_key(__ldcg(&keys[pos])), smax);
-    const uint4* row = reinterpret_cast<const uint4*>(P.k + (u.k_row0 + pos) * kHeadDim);
-    float ss = 0.f;
+  // candidate keys row-major in shared memory (slot order = position order); a
+  // half-warp copies one 256-byte row, coalesced
+  {
+    constexpr int kRows = NT / (NT / 32 * 2);      // rows per half-warp: 8 (NT=256) or 16 (NT=512)
+    uint4 xr[kRows];
 #pragma unroll
-    for (int j = 0; j < kChunks; ++j) {
-      const uint4 x = __ldg(row + j);
-      kch[j * kMaxCand + tid] = x;
-      const uint32_t w4[4] = {x.x, x.y, x.z, x.w};
+    for (int q = 0; q < kRows; ++q) {
+      const int r = (q * (NT / 32) + warp) * 2 + (lane >> 4);
+      xr[q] = make_uint4(0, 0, 0, 0);
+      if (r < C) {
+        const uint4* src = reinterpret_cast<const uint4*>(P.k + (u.k_row0 + spos[r]) * kHeadDim);
+        xr[q] = __ldg(src + (lane & 15));
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < kRows; ++q) {
+      const int r = (q * (NT / 32) + warp) * 2 + (lane >> 4);
+      if (r < C) krow[r * kChunks + (lane & 15)] = xr[q];
+      const uint32_t w4[4] = {xr[q].x, xr[q].y, xr[q].z, xr[q].w};
+      float ss = 0.f;
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const float lo = __uint_as_float(w4[e] << 16);
@@ -214,85 +350,151 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const __grid_con
         ss = fmaf(lo, lo, ss);
         ss = fmaf(hi, hi, ss);
       }
+#pragma unroll
+      for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+      if (r < C && (lane & 15) == 0) inv[r] = ss > 0.f ? __fdiv_rn(1.0f, sqrtf(ss)) : 0.f;
     }
-    inv[tid] = ss > 0.f ? __fdiv_rn(1.0f, sqrtf(ss)) : 0.f;
   }
   __syncthreads();
 
-  // 5. greedy admissions
-  const float my_st = tid < C ? st[tid] : 0.f;
-  const float my_inv = tid < C ? inv[tid] : 0.f;
+  // 5. greedy admissions. Lane (g, t) of a warp owns slot
+  //    warp*32 + 16*(t>>1) + g + 8*(t&1); the warp's 32 candidate keys stay in
+  //    registers as mma.m16n8k16 A fragments, and every admission computes the
+  //    32 dot products with the admitted key by 16 tensor-core MMAs (bf16 products,
+  //    fp32 accumulation) with that key replicated in the 8 columns of B.
+  const int g = lane >> 2, tq = lane & 3;
+  const int slot = warp * 32 + 16 * (tq >> 1) + g + 8 * (tq & 1);
+  bool active = slot < C;
+  float corr = 0.f;
+  const float my_st = active ? __fdiv_rn(unord_key(__ldcg(&keys[spos[slot]])), smax) : 0.f;
+  const float my_inv = active ? inv[slot] : 0.f;
+  const uint32_t* kw = reinterpret_cast<const uint32_t*>(krow);   // 64 words per row
+  uint32_t afr[2][8][4];
+#pragma unroll
+  for (int m = 0; m < 2; ++m) {
+    const int r0 = warp * 32 + 16 * m + g, r1 = r0 + 8;
+#pragma unroll
+    for (int s8 = 0; s8 < 8; ++s8) {
+      afr[m][s8][0] = r0 < C ? kw[r0 * 64 + 8 * s8 + tq] : 0u;
+      afr[m][s8][1] = r1 < C ? kw[r1 * 64 + 8 * s8 + tq] : 0u;
+      afr[m][s8][2] = r0 < C ? kw[r0 * 64 + 8 * s8 + tq + 4] : 0u;
+      afr[m][s8][3] = r1 < C ? kw[r1 * 64 + 8 * s8 + tq + 4] : 0u;
+    }
+  }
   int32_t* order = P.order ? P.order + u.unit * B : nullptr;
   float* margins = P.margins ? P.margins + u.unit * B : nullptr;
   for (int t = 0; t < nsel; ++t) {
-    unsigned long long b1 = 0, b2 = 0;
-    if (!mine_taken) {
-      const float v = fmaf(lambda2, corr, my_st);
-      b1 = (static_cast<unsigned long long>(ord_key(v)) << 32) |
-           static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(tid));
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-      const unsigned long long o1 = __shfl_xor_sync(0xffffffffu, b1, o);
-      const unsigned long long o2 = __shfl_xor_sync(0xffffffffu, b2, o);
-      top2_merge(b1, b2, o1, o2);
-    }
+    const uint32_t key = active ? ord_key(fmaf(lambda2, corr, my_st)) : 0u;
+    const uint32_t wmax = __reduce_max_sync(0xffffffffu, key);
+    const uint32_t wslot = __reduce_min_sync(0xffffffffu, (active && key == wmax) ? slot : 0xFFFFFFFFu);
+    const uint32_t wsec = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(slot) == wslot ? 0u : key);
     if (lane == 0) {
-      sh.red[t & 1][warp][0] = b1;
-      sh.red[t & 1][warp][1] = b2;
+      sh.red[t & 1][warp][0] = wmax;
+      sh.red[t & 1][warp][1] = wslot;
+      sh.red[t & 1][warp][2] = wsec;
     }
     __syncthreads();
-    unsigned long long f1 = 0, f2 = 0;
+    uint32_t best = 0, bslot = 0xFFFFFFFFu, sec = 0;
 #pragma unroll
-    for (int w = 0; w < kSelThreads / 32; ++w) top2_merge(f1, f2, sh.red[t & 1][w][0], sh.red[t & 1][w][1]);
-    const int js = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(f1 & 0xFFFFFFFFull));
+    for (int w = 0; w < NT / 32; ++w) {
+      const uint32_t k = sh.red[t & 1][w][0], sl = sh.red[t & 1][w][1], k2 = sh.red[t & 1][w][2];
+      if (k > best || (k == best && sl < bslot)) {
+        sec = max(sec, best);
+        best = k;
+        bslot = sl;
+      } else {
+        sec = max(sec, k);
+      }
+      sec = max(sec, k2);
+    }
+    const int js = static_cast<int>(bslot);
     if (tid == 0) {
       if (order) order[t] = spos[js];
-      if (margins) {
-        const float vb = unord_key(static_cast<uint32_t>(f1 >> 32));
-        margins[t] = f2 ? vb - unord_key(static_cast<uint32_t>(f2 >> 32)) : INFINITY;
+      if (margins) margins[t] = sec ? unord_key(best) - unord_key(sec) : INFINITY;
+    }
+    if (slot == js) active = false;
+    // dots of the warp's candidates with the admitted key (two accumulation chains
+    // per tile: even and odd k-steps)
+    float d[2][2][4];
+#pragma unroll
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) d[m][c][e] = 0.f;
+    uint32_t bf[8][2];
+#pragma unroll
+    for (int s8 = 0; s8 < 8; ++s8) {
+      bf[s8][0] = kw[js * 64 + 8 * s8 + tq];
+      bf[s8][1] = kw[js * 64 + 8 * s8 + tq + 4];
+    }
+#pragma unroll
+    for (int s8 = 0; s8 < 8; ++s8) {
+#pragma unroll
+      for (int m = 0; m < 2; ++m) {
+        float* dd = d[m][s8 & 1];
+        asm volatile(
+            "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+            "{%8,%9}, {%0,%1,%2,%3};"
+            : "+f"(dd[0]), "+f"(dd[1]), "+f"(dd[2]), "+f"(dd[3])
+            : "r"(afr[m][s8][0]), "r"(afr[m][s8][1]), "r"(afr[m][s8][2]), "r"(afr[m][s8][3]),
+              "r"(bf[s8][0]), "r"(bf[s8][1]));
       }
     }
-    if (tid == js) mine_taken = true;
-    if (!mine_taken) {
-      float dot = 0.f;
-#pragma unroll
-      for (int j = 0; j < kChunks; ++j) {
-        const uint4 a = kch[j * kMaxCand + tid];
-        const uint4 b = kch[j * kMaxCand + js];
-        const uint32_t aw[4] = {a.x, a.y, a.z, a.w};
-        const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          dot = fmaf(__uint_as_float(aw[e] << 16), __uint_as_float(bw[e] << 16), dot);
-          dot = fmaf(__uint_as_float(aw[e] & 0xFFFF0000u), __uint_as_float(bw[e] & 0xFFFF0000u), dot);
-        }
-      }
-      corr = fmaxf(corr, dot * my_inv * inv[js]);
-    }
+    // rows g (element 0) and g + 8 (element 2) of tile t>>1; every column holds the same dot
+    const int mt = tq >> 1, el = (tq & 1) ? 2 : 0;
+    const float dot = d[mt][0][el] + d[mt][1][el];
+    if (active) corr = fmaxf(corr, dot * my_inv * inv[js]);
   }
 
   // 6. admitted positions in ascending order, then -1
-  const bool sel = tid < C && mine_taken;
+  // slot s is admitted iff its owner went inactive; mark, then rank in slot order
+  __syncthreads();
+  if (slot < C) cpos[slot] = active ? 0 : 1;
+  __syncthreads();
+  const bool sel = tid < C && cpos[tid] != 0;
   uint32_t tot;
-  const uint32_t rank = block_excl_count(sel, sh, &tot);
+  const uint32_t rank = block_excl_count<NT>(sel, sh, &tot);
   int32_t* out = P.indices + u.unit * B;
   if (sel) out[rank] = spos[tid];
-  for (int r = nsel + tid; r < B; r += kSelThreads) out[r] = -1;
+  for (int r = nsel + tid; r < B; r += NT) out[r] = -1;
   if (order)
-    for (int r = nsel + tid; r < B; r += kSelThreads) order[r] = -1;
+    for (int r = nsel + tid; r < B; r += NT) order[r] = -1;
   if (margins)
-    for (int r = nsel + tid; r < B; r += kSelThreads) margins[r] = 0.f;
+    for (int r = nsel + tid; r < B; r += NT) margins[r] = 0.f;
 }
+
+template <int NT>
+constexpr size_t select_smem() {
+  // candidate keys (also reused for the pooling tiles and the histogram) + 4 arrays
+  return kChunks * NT * sizeof(uint4) + 4 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
+}
+static_assert(kChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histogram fits");
+static_assert(kChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
+              "pool tiles fit");
+static_assert(kChunks * 256 * sizeof(uint4) >= kTieCap * sizeof(int32_t), "tie list fits");
 
 }  // namespace
 
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {
-  const size_t dyn = kChunks * kMaxCand * sizeof(uint4) + 4 * kMaxCand * sizeof(int32_t);
-  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(dyn));
-  if (e != cudaSuccess) return e;
-  select_kernel<<<static_cast<unsigned>(plan.geo.n_units), kSelThreads, dyn, stream>>>(p);
+  // pool size bound: the largest C over the requests
+  int max_lc = 0;
+  for (int r = 0; r < plan.geo.n_req; ++r) max_lc = max(max_lc, plan.geo.req_len[r] - plan.geo.window);
+  const int cmax = p.cand_factor == 0 ? max_lc : min(p.cand_factor * p.budget, max_lc);
+  const unsigned grid = static_cast<unsigned>(plan.geo.n_units);
+  if (cmax <= 256) {
+    constexpr size_t smem = select_smem<256>();
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    select_kernel<256><<<grid, 256, smem, stream>>>(p);
+  } else {
+    constexpr size_t smem = select_smem<512>();
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<512>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    select_kernel<512><<<grid, 512, smem, stream>>>(p);
+  }
   return cudaGetLastError();
 }
 
