@@ -129,11 +129,10 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   kve::WsLayout& w = plan->ws;
   w.hdr = 0;
   w.counts = 256;
-  w.flags = align_up(w.counts + 4 * units, 256);
-  w.clear_end = align_up(w.flags + 4 * units, 256);
+  w.beta = align_up(w.counts + 4 * units, 256);
+  w.clear_end = align_up(w.beta + sizeof(uint64_t) * kMaxRows * units, 256);
   w.partial = w.clear_end;
-  w.beta = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
-  w.keys = align_up(w.beta + sizeof(float) * kMaxRows * units, 256);
+  w.keys = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
   w.total = align_up(w.keys + sizeof(uint32_t) * units_per_req * off, 256);
   if (workspace_bytes) *workspace_bytes = w.total;
   *plan_out = plan;
@@ -178,9 +177,8 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
   p.err = reinterpret_cast<uint32_t*>(w);
   p.claim = reinterpret_cast<uint32_t*>(w + 4);
   p.counts = reinterpret_cast<uint32_t*>(w + plan->ws.counts);
-  p.flags = reinterpret_cast<uint32_t*>(w + plan->ws.flags);
   p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
-  p.beta = reinterpret_cast<float*>(w + plan->ws.beta);
+  p.beta = reinterpret_cast<unsigned long long*>(w + plan->ws.beta);
   return kve::launch_score(*plan, tm_q, tm_k, p, sms, st) == cudaSuccess ? KVE_OK : KVE_ECUDA;
 }
 

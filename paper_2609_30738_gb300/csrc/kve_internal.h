@@ -75,10 +75,9 @@ __host__ __device__ inline int64_t item_unit(const Geometry& g, int64_t p, int32
 struct WsLayout {
   size_t hdr;        // uint32 err, uint32 claim, padding to 256 B
   size_t counts;     // uint32 [n_units]  row-statistics arrivals per unit
-  size_t flags;      // uint32 [n_units]  merged statistics ready
+  size_t beta;       // uint64 [n_units][kMaxRows]  (log2 softmax normaliser, ready tag)
   size_t clear_end;  // bytes from 0 cleared before each score call
   size_t partial;    // float2 [n_items][kMaxRows]  per-item (max, sum) in log2 units
-  size_t beta;       // float  [n_units][kMaxRows]  log2 softmax normaliser per row
   size_t keys;       // uint32 [sum of unit lengths]  ordered base scores (select)
   size_t total;
 };
@@ -94,9 +93,8 @@ struct ScoreParams {
   uint32_t* err;
   uint32_t* claim;
   uint32_t* counts;
-  uint32_t* flags;
   float2* partial;
-  float* beta;
+  unsigned long long* beta;   // low word: beta bits, high word: 1 once written
 };
 
 struct SelectParams {

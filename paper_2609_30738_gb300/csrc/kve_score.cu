@@ -300,11 +300,19 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
                                               const UnitInfo& u, int64_t p, uint32_t slot) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
+  float2 mz[4];
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const int row = lane + 32 * k;
-    const float2 mz = merge_mz(ctl.comb[slot][0][row], ctl.comb[slot][1][row]);
-    if (row < n) P.partial[p * kMaxRows + row] = mz;
+    mz[k] = merge_mz(ctl.comb[slot][0][row], ctl.comb[slot][1][row]);
+  }
+  // the slot's shared data is in registers: hand the slot back to the producer
+  __syncwarp();
+  if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int row = lane + 32 * k;
+    if (row < n) P.partial[p * kMaxRows + row] = mz[k];
   }
   __threadfence();
   __syncwarp();
@@ -319,12 +327,12 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
     float2 acc[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) acc[k] = make_float2(-INFINITY, 0.f);
-    for (int s0 = 0; s0 < u.splits; s0 += 16) {
-      float2 pz[4][16];
+    for (int s0 = 0; s0 < u.splits; s0 += 8) {
+      float2 pz[4][8];
 #pragma unroll
       for (int k = 0; k < 4; ++k)
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
+        for (int j = 0; j < 8; ++j) {
           const int row = lane + 32 * k;
           pz[k][j] = (s0 + j < u.splits && row < n)
                          ? __ldcg(&P.partial[(u.item0 + s0 + j) * kMaxRows + row])
@@ -333,48 +341,54 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
 #pragma unroll
       for (int k = 0; k < 4; ++k)
 #pragma unroll
-        for (int j = 0; j < 16; ++j) acc[k] = merge_mz(acc[k], pz[k][j]);
+        for (int j = 0; j < 8; ++j) acc[k] = merge_mz(acc[k], pz[k][j]);
     }
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int row = lane + 32 * k;
-      if (row < n) __stcg(&P.beta[u.unit * kMaxRows + row], acc[k].x + lg2(acc[k].y));
+      if (row < n) {
+        // one 64-bit store: a reader sees either the cleared word or (beta, 1)
+        const float b = acc[k].x + lg2(acc[k].y);
+        const unsigned long long word =
+            (1ull << 32) | static_cast<unsigned long long>(__float_as_uint(b));
+        __stcg(&P.beta[u.unit * kMaxRows + row], word);
+      }
     }
-    __threadfence();
-    __syncwarp();
-    if (lane == 0) st_release_gpu(&P.flags[u.unit], 1u);
   }
   return true;
 }
 
-// Phase-1 item: wait for the unit's merged statistics and stage -beta.
+// Phase-1 item: wait for the unit's merged statistics and stage -beta. Each row's
+// normaliser carries its own ready tag, so one round of loads both checks and
+// fetches it.
 __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ctl,
                                               const UnitInfo& u, uint32_t slot) {
   const int lane = threadIdx.x & 31;
-  int ok = 1;
-  if (lane == 0) {
-    const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
-    const volatile uint32_t* errw = P.err;
-    uint32_t ns = 32;
-    while (ld_acquire_gpu(&P.flags[u.unit]) == 0u) {
-      if (*errw != 0u || ctl.abort || global_timer_ns() > deadline) {
-        ok = 0;
-        break;
-      }
-      __nanosleep(ns);
-      if (ns < 512) ns *= 2;
-    }
-  }
-  ok = __shfl_sync(0xffffffffu, ok, 0);
-  if (!ok) return false;
-  __syncwarp();   // orders every lane's loads after lane 0's acquire
   const int n = P.g.n_rows;
-  float4 b;
   const int r0 = 4 * lane;
-  b.x = r0 + 0 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 0]) : -INFINITY;
-  b.y = r0 + 1 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 1]) : -INFINITY;
-  b.z = r0 + 2 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 2]) : -INFINITY;
-  b.w = r0 + 3 < n ? -__ldcg(&P.beta[u.unit * kMaxRows + r0 + 3]) : -INFINITY;
+  const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
+  const volatile uint32_t* errw = P.err;
+  uint32_t ns = 32;
+  unsigned long long w[4];
+  for (;;) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      w[k] = (r0 + k < n) ? __ldcg(&P.beta[u.unit * kMaxRows + r0 + k]) : (1ull << 32);
+    bool ready = true;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
+    if (__all_sync(0xffffffffu, ready)) break;
+    int give_up = 0;
+    if (lane == 0) give_up = (*errw != 0u || ctl.abort || global_timer_ns() > deadline) ? 1 : 0;
+    if (__shfl_sync(0xffffffffu, give_up, 0)) return false;
+    __nanosleep(ns);
+    if (ns < 512) ns *= 2;
+  }
+  float4 b;
+  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
+  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
+  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
+  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
   reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
   return true;
 }
@@ -579,18 +593,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (cl.phase == 0) {
         if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);      // nothing to stage
         ok = warp_wait(&ctl.pub_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
-             sync_rowstats(P, ctl, u, cl.p, slot);
+             sync_rowstats(P, ctl, u, cl.p, slot);            // hands the slot back early
       } else {
         ok = sync_colstats(P, ctl, u, slot);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);
+        if (lane == 0) {
+          mbar_arrive(&ctl.beta_full[slot]);
+          mbar_arrive(&ctl.item_empty[slot]);
+        }
       }
       if (!ok) {
         set_error(P, ctl, 1u);
         break;
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
       ++it;
     }
   } else {
