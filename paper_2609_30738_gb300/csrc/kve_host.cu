@@ -129,7 +129,8 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   kve::WsLayout& w = plan->ws;
   w.hdr = 0;
   w.counts = 256;
-  w.beta = align_up(w.counts + 4 * units, 256);
+  w.done = align_up(w.counts + 4 * units, 256);
+  w.beta = align_up(w.done + 4 * units, 256);
   w.clear_end = align_up(w.beta + sizeof(uint64_t) * kMaxRows * units, 256);
   w.partial = w.clear_end;
   w.keys = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
@@ -167,16 +168,15 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
   std::memset(&p, 0, sizeof(p));
   p.g = g;
   p.alpha = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
-  int max_splits = 1;
-  for (int r = 0; r < g.n_req; ++r) max_splits = std::max(max_splits, g.req_splits[r]);
-  p.lag = std::min<int64_t>(g.n_items, static_cast<int64_t>(max_splits) + 2 * sms);
   p.wait_limit_ns = plan->wait_limit_ns;
   p.fault = plan->fault;
   p.mu = mu;
   p.sigma = sigma;
   p.err = reinterpret_cast<uint32_t*>(w);
-  p.claim = reinterpret_cast<uint32_t*>(w + 4);
+  p.claim1 = reinterpret_cast<uint32_t*>(w + 4);
+  p.claim2 = reinterpret_cast<uint32_t*>(w + 8);
   p.counts = reinterpret_cast<uint32_t*>(w + plan->ws.counts);
+  p.done = reinterpret_cast<uint32_t*>(w + plan->ws.done);
   p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
   p.beta = reinterpret_cast<unsigned long long*>(w + plan->ws.beta);
   return kve::launch_score(*plan, tm_q, tm_k, p, sms, st) == cudaSuccess ? KVE_OK : KVE_ECUDA;

@@ -73,8 +73,9 @@ __host__ __device__ inline int64_t item_unit(const Geometry& g, int64_t p, int32
 
 // Workspace layout (byte offsets from the caller's workspace pointer).
 struct WsLayout {
-  size_t hdr;        // uint32 err, uint32 claim, padding to 256 B
+  size_t hdr;        // uint32 err, uint32 row-item claims, uint32 column-item claims
   size_t counts;     // uint32 [n_units]  row-statistics arrivals per unit
+  size_t done;       // uint32 [n_units]  1 once the unit's normalisers are written
   size_t beta;       // uint64 [n_units][kMaxRows]  (log2 softmax normaliser, ready tag)
   size_t clear_end;  // bytes from 0 cleared before each score call
   size_t partial;    // float2 [n_items][kMaxRows]  per-item (max, sum) in log2 units
@@ -85,14 +86,15 @@ struct WsLayout {
 struct ScoreParams {
   Geometry g;
   float alpha;               // log2(e) / sqrt(d)
-  int64_t lag;               // row-statistics items issued before the first column item
   uint64_t wait_limit_ns;
   int32_t fault;             // test hook: 1 = unit 0 never publishes its statistics
   float* mu;
   float* sigma;
   uint32_t* err;
-  uint32_t* claim;
+  uint32_t* claim1;          // next row-statistics item
+  uint32_t* claim2;          // next column-statistics item
   uint32_t* counts;
+  uint32_t* done;
   float2* partial;
   unsigned long long* beta;   // low word: beta bits, high word: 1 once written
 };

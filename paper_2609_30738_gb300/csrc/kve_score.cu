@@ -17,11 +17,15 @@
 //                               epilogue thread owns one key, forms
 //                               A = 2^(alpha*l - beta_r) for its n rows and reduces
 //                               them to mu and sigma in registers (two passes).
-// Items are claimed in a global order in which every phase-0 item of a unit comes
-// before any phase-1 item of it, and phase-1 items trail phase-0 items by `lag`
-// items so that their K tiles are still in L2. A CTA processes its claims in
-// order, so a phase-1 item only ever waits for phase-0 items claimed before it;
-// every wait is bounded and a timeout is reported as KVE_ETIMEOUT.
+// Work is claimed from two queues, both in unit order. A CTA's producer holds one
+// claimed phase-1 item and pushes it into the CTA's pipeline only once its unit's
+// statistics are merged (a relaxed poll of the unit's done flag, overlapped with
+// the loads of the current item); until then it claims phase-0 items. Nothing
+// waits on another CTA while phase-0 work remains, so the schedule needs neither an
+// ordering argument nor co-residency, and a phase-1 item re-reads its K tiles about
+// one merge latency after they were streamed, while they are still in L2. The
+// final waits (no phase-0 work left) are bounded and a timeout is reported as
+// KVE_ETIMEOUT.
 //
 // Roles: warp 0 claims items and issues TMA loads; warp 1 owns TMEM and issues the
 // MMAs; warp 2 (sync) does all cross-CTA work in claim order -- it publishes the
@@ -75,22 +79,15 @@ struct Claim {
   int64_t p;
 };
 
-__device__ __forceinline__ Claim decode_claim(int64_t c, int64_t n1, int64_t lag) {
+// Ring entry: item index in the low bits, phase in bit 62; -1 ends the work.
+__device__ __forceinline__ int64_t encode_claim(int phase, int64_t p) {
+  return p | (static_cast<int64_t>(phase) << 62);
+}
+
+__device__ __forceinline__ Claim decode_claim(int64_t c) {
   Claim k;
-  if (c < lag) {
-    k.phase = 0;
-    k.p = c;
-    return k;
-  }
-  const int64_t j = c - lag;
-  const int64_t inter = 2 * (n1 - lag);
-  if (j < inter) {
-    k.phase = static_cast<int>(j & 1);
-    k.p = (j & 1) ? (j >> 1) : lag + (j >> 1);
-  } else {
-    k.phase = 1;
-    k.p = j - (n1 - lag);
-  }
+  k.phase = static_cast<int>((c >> 62) & 1);
+  k.p = c & ((int64_t(1) << 62) - 1);
   return k;
 }
 
@@ -354,6 +351,9 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
         __stcg(&P.beta[u.unit * kMaxRows + row], word);
       }
     }
+    __threadfence();
+    __syncwarp();
+    if (lane == 0) st_release_gpu(&P.done[u.unit], 1u);   // hint for the producers
   }
   return true;
 }
@@ -409,7 +409,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int64_t n1 = P.g.n_items;
-  const int64_t total_claims = 2 * n1;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kQBufs; ++i) { mbar_init(&ctl.q_full[i], 1); mbar_init(&ctl.q_empty[i], 1); }
@@ -444,24 +443,104 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_keep = l2_policy_evict_last();
       const uint64_t pol_drop = l2_policy_evict_first();
       bool ok = true;
-      // the next claim is requested one item ahead so that its round trip overlaps
-      // the loads of the current item (claims are still processed in order)
-      uint32_t next = atomicAdd(P.claim, 1u);
+      // Row items are claimed one ahead. Column items are claimed only when the unit
+      // at the head of the column queue is ready: the head index and its unit's done
+      // flag are polled with relaxed loads whose values are used one item later. A
+      // claim that raced past the ready front is held until its unit is ready.
+      const volatile uint32_t* errw = P.err;
+      int s2;
+      int64_t p1 = atomicAdd(P.claim1, 1u);
+      int64_t held = -1;                               // claimed, not yet ready
+      int64_t head = 0;                                // queue head the flag refers to
+      uint32_t head_ready = 0;                         // done flag of head's unit
+      int64_t peek = 0;                                // newest peek of the queue head
+      uint32_t held_ready = 0;
       for (;;) {
-        int64_t c = ctl.abort ? total_claims : static_cast<int64_t>(next);
-        if (c > total_claims) c = total_claims;
-        if (c < total_claims) next = atomicAdd(P.claim, 1u);
+        Claim cl;
+        bool have = false;
+        if (ctl.abort) {
+          have = false;
+        } else if (held >= 0 && held_ready) {
+          cl.phase = 1;
+          cl.p = held;
+          have = true;
+          held = -1;
+        } else if (held < 0 && head < n1 && head_ready) {
+          const int64_t q = atomicAdd(P.claim2, 1u);
+          if (q < n1) {
+            if (item_unit(P.g, q, &s2) == item_unit(P.g, head, &s2)) {
+              cl.phase = 1;
+              cl.p = q;
+              have = true;
+            } else {
+              held = q;
+              held_ready = 0;
+            }
+          }
+        }
+        if (!have && !ctl.abort && p1 < n1) {
+          cl.phase = 0;
+          cl.p = p1;
+          have = true;
+          p1 = atomicAdd(P.claim1, 1u);
+        }
+        if (!have && !ctl.abort) {
+          // no row work left: wait (bounded) for column work to become ready
+          const int64_t h = ld_volatile_u32(P.claim2);
+          if (held < 0 && h >= n1) {
+            have = false;                              // all work is claimed: finish
+          } else {
+            const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
+            uint32_t ns = 64;
+            bool ready = false;
+            for (;;) {
+              const int64_t x = held >= 0 ? held : static_cast<int64_t>(ld_volatile_u32(P.claim2));
+              if (x >= n1) break;
+              if (ld_volatile_u32(&P.done[item_unit(P.g, x, &s2)])) {
+                ready = true;
+                break;
+              }
+              if (*errw != 0u || ctl.abort || global_timer_ns() > deadline) break;
+              __nanosleep(ns);
+              if (ns < 1024) ns *= 2;
+            }
+            if (held >= 0) {
+              if (!ready) {
+                ok = false;
+                break;
+              }
+              held_ready = 1;
+            } else {
+              if (!ready && ld_volatile_u32(P.claim2) < n1) {
+                ok = false;
+                break;
+              }
+              head = ld_volatile_u32(P.claim2);
+              peek = head;
+              head_ready = ready ? 1u : 0u;
+            }
+            continue;
+          }
+        }
+        // refresh the polls, consumed at the next decision: the done flag of the
+        // head peeked last time, and an independent new peek of the head
+        if (held >= 0) {
+          held_ready = ld_volatile_u32(&P.done[item_unit(P.g, held, &s2)]);
+        } else {
+          head = peek;
+          head_ready = head < n1 ? ld_volatile_u32(&P.done[item_unit(P.g, head, &s2)]) : 0u;
+          peek = ld_volatile_u32(P.claim2);
+        }
         const uint32_t slot = it % kItemSlots;
         if (!mbar_wait(&ctl.item_empty[slot], ((it / kItemSlots) & 1u) ^ 1u,
                        global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
           ok = false;
           break;
         }
-        ctl.item_ring[slot] = (c >= total_claims) ? -1 : c;
+        ctl.item_ring[slot] = have ? encode_claim(cl.phase, cl.p) : -1;
         mbar_arrive(&ctl.item_full[slot]);
         ++it;
-        if (c >= total_claims) break;
-        const Claim cl = decode_claim(c, n1, P.lag);
+        if (!have) break;
         int split;
         const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
         const uint32_t qb = qi % kQBufs;
@@ -524,7 +603,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_arrive(&ctl.item_empty[slot]);
         ++it;
         if (c < 0) break;
-        const Claim cl = decode_claim(c, n1, P.lag);
+        const Claim cl = decode_claim(c);
         int split;
         const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
         const uint32_t qb = qi % kQBufs;
@@ -586,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const int64_t c = ctl.item_ring[slot];
       if (c < 0) break;
-      const Claim cl = decode_claim(c, n1, P.lag);
+      const Claim cl = decode_claim(c);
       int split;
       const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
       bool ok;
@@ -620,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const int64_t c = ctl.item_ring[slot];
       if (c < 0) break;
-      const Claim cl = decode_claim(c, n1, P.lag);
+      const Claim cl = decode_claim(c);
       int split;
       const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
       bool ok;
@@ -660,8 +739,8 @@ cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CU
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kDynSmem));
   if (e != cudaSuccess) return e;
-  const int64_t claims = 2 * p.g.n_items;
-  const int grid = static_cast<int>(claims < num_sms ? claims : num_sms);
+  const int64_t items = p.g.n_items;
+  const int grid = static_cast<int>(items < num_sms ? items : num_sms);
   fn<<<grid, kThreads, kDynSmem, stream>>>(tm_q, tm_k, p);
   return cudaGetLastError();
 }
