@@ -1,5 +1,6 @@
 // Host side of the kv_evict C ABI: plan validation and work geometry, workspace
 // layout, TMA descriptor encoding and the launches of the three kernels.
+#include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -16,7 +17,8 @@ using kve::kHeadDim;
 using kve::kMaxLayers;
 using kve::kMaxReq;
 using kve::kMaxRows;
-using kve::kSplitKeys;
+using kve::kSplitTiles;
+using kve::kTileKeys;
 
 constexpr uint64_t kDefaultWaitNs = 2000000000ull;   // 2 s
 constexpr int kMaxCand = 512;
@@ -60,6 +62,37 @@ int device_sms() {
   return sms;
 }
 
+// Score items per unit for a unit of T tiles. Items hold at most kSplitTiles tiles.
+// The score kernel deals items to its CTAs round-robin, one round = one item per CTA,
+// so a split count that divides the CTA count (or is a multiple of it) makes every
+// round hold whole units; up to twice the minimum count is accepted for that.
+int32_t choose_splits(int64_t T, int64_t ctas) {
+  const int64_t kmin = (T + kSplitTiles - 1) / kSplitTiles;
+  const int64_t kmax = std::min<int64_t>(T, 2 * kmin);
+  for (int64_t k = kmin; ctas > 0 && k <= kmax; ++k)
+    if (ctas % k == 0 || k % ctas == 0) return static_cast<int32_t>(k);
+  return static_cast<int32_t>(kmin);
+}
+
+// Rounds a CTA's phase-1 item must trail its phase-0 item in the score kernel: one
+// more than the most rounds any unit's items span, so that every unit's row
+// statistics are complete (or only one round of work away) when its first phase-1
+// item comes up. Any lag >= the span is free of circular waits.
+int32_t score_lag(const kve::Geometry& g, int64_t ctas) {
+  int64_t span = 0;
+  const int64_t units_per_req = static_cast<int64_t>(g.num_layers) * g.hkv;
+  for (int r = 0; r < g.n_req; ++r) {
+    const int64_t k = g.req_splits[r];
+    // (first item) mod ctas repeats with period ctas / gcd(k, ctas) <= ctas
+    const int64_t n = std::min<int64_t>(units_per_req, ctas);
+    for (int64_t ul = 0; ul < n; ++ul) {
+      const int64_t a = g.req_item_base[r] + ul * k;
+      span = std::max<int64_t>(span, (a + k - 1) / ctas - a / ctas);
+    }
+  }
+  return static_cast<int32_t>(span + 1);
+}
+
 }  // namespace
 
 extern "C" {
@@ -95,6 +128,11 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   g.n_rows = G * c.window;
   int64_t off = 0, units = 0, items = 0, max_lc = 0;
   const int64_t units_per_req = static_cast<int64_t>(c.num_layers) * c.num_kv_heads;
+  int ctas = device_sms();
+  if (ctas <= 0) {
+    cudaGetLastError();
+    ctas = 152;   // no device visible: plan for a full GB300
+  }
   for (int r = 0; r < n_req; ++r) {
     const int64_t L = seq_lens[r];
     if (L <= c.window || L > (int64_t(1) << 30)) {
@@ -103,7 +141,8 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
     }
     g.req_len[r] = static_cast<int32_t>(L);
     g.req_tok_off[r] = off;
-    g.req_splits[r] = static_cast<int32_t>((L + kSplitKeys - 1) / kSplitKeys);
+    g.req_tiles[r] = static_cast<int32_t>((L + kTileKeys - 1) / kTileKeys);
+    g.req_splits[r] = choose_splits(g.req_tiles[r], ctas);
     g.req_unit_base[r] = units;
     g.req_item_base[r] = items;
     off += L;
@@ -129,8 +168,7 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   kve::WsLayout& w = plan->ws;
   w.hdr = 0;
   w.counts = 256;
-  w.done = align_up(w.counts + 4 * units, 256);
-  w.beta = align_up(w.done + 4 * units, 256);
+  w.beta = align_up(w.counts + 4 * units, 256);
   w.clear_end = align_up(w.beta + sizeof(uint64_t) * kMaxRows * units, 256);
   w.partial = w.clear_end;
   w.keys = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
@@ -173,13 +211,13 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
   p.mu = mu;
   p.sigma = sigma;
   p.err = reinterpret_cast<uint32_t*>(w);
-  p.claim1 = reinterpret_cast<uint32_t*>(w + 4);
-  p.claim2 = reinterpret_cast<uint32_t*>(w + 8);
   p.counts = reinterpret_cast<uint32_t*>(w + plan->ws.counts);
-  p.done = reinterpret_cast<uint32_t*>(w + plan->ws.done);
   p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
   p.beta = reinterpret_cast<unsigned long long*>(w + plan->ws.beta);
-  return kve::launch_score(*plan, tm_q, tm_k, p, sms, st) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+  const int64_t ctas = std::min<int64_t>(sms, g.n_items);
+  p.lag = score_lag(g, ctas);
+  return kve::launch_score(*plan, tm_q, tm_k, p, static_cast<int>(ctas), st) == cudaSuccess ? KVE_OK
+                                                                                        : KVE_ECUDA;
 }
 
 kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,

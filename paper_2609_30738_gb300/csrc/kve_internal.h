@@ -13,8 +13,7 @@ namespace kve {
 
 constexpr int kHeadDim = 128;      // d supported by this build
 constexpr int kTileKeys = 128;     // keys per MMA tile (one TMEM accumulator)
-constexpr int kSplitTiles = 8;     // tiles per work item
-constexpr int kSplitKeys = kTileKeys * kSplitTiles;
+constexpr int kSplitTiles = 8;     // most tiles in one work item
 constexpr int kMaxRows = 128;      // n = G*W window rows per unit, padded to one M tile
 constexpr int kMaxReq = 64;        // requests per call
 constexpr int kMaxLayers = 256;    // layers per call (lambda arrays ride in kernel params)
@@ -27,7 +26,8 @@ struct Geometry {
   int64_t n_items;                      // score work items (sum over units of splits)
   int32_t req_len[kMaxReq];             // L_r
   int64_t req_tok_off[kMaxReq];         // off_r
-  int32_t req_splits[kMaxReq];          // ceil(L_r / kSplitKeys)
+  int32_t req_tiles[kMaxReq];           // ceil(L_r / kTileKeys)
+  int32_t req_splits[kMaxReq];          // work items per unit (<= req_tiles)
   int64_t req_unit_base[kMaxReq + 1];   // first unit of request r
   int64_t req_item_base[kMaxReq + 1];   // first item of request r
 };
@@ -36,7 +36,9 @@ struct UnitInfo {
   int64_t unit;        // (r, l, h) flattened, request-major
   int32_t r, layer, h;
   int32_t L;           // prefix length
+  int32_t tiles;       // ceil(L / kTileKeys)
   int32_t splits;      // items of this unit
+  int64_t local;       // unit index within its request
   int64_t q_row0;      // first window row in q_win viewed as [rows][d]
   int64_t k_row0;      // first key row in k viewed as [rows][d]
   int64_t mu_off;      // first element of this unit in mu / sigma
@@ -53,7 +55,9 @@ __host__ __device__ inline UnitInfo unit_info(const Geometry& g, int64_t unit) {
   u.layer = static_cast<int32_t>(local / g.hkv);
   u.h = static_cast<int32_t>(local % g.hkv);
   u.L = g.req_len[r];
+  u.tiles = g.req_tiles[r];
   u.splits = g.req_splits[r];
+  u.local = local;
   u.q_row0 = ((static_cast<int64_t>(u.layer) * g.n_req + r) * g.hq +
               static_cast<int64_t>(u.h) * g.group) * g.window;
   u.k_row0 = (static_cast<int64_t>(u.layer) * g.hkv + u.h) * g.total_tokens + g.req_tok_off[r];
@@ -71,11 +75,21 @@ __host__ __device__ inline int64_t item_unit(const Geometry& g, int64_t p, int32
   return g.req_unit_base[r] + local / g.req_splits[r];
 }
 
+// Tiles [*t0, *t0 + *nt) of item `split` of unit u. The unit's tiles are cut into
+// u.splits near-equal runs; the run index is rotated by the unit index so that a
+// CTA that always holds the same split index does not always get the longer runs.
+__host__ __device__ inline void item_range(const UnitInfo& u, int split, int* t0, int* nt) {
+  const int64_t s = (split + u.local) % u.splits;
+  const int64_t a = s * u.tiles / u.splits;
+  const int64_t b = (s + 1) * u.tiles / u.splits;
+  *t0 = static_cast<int>(a);
+  *nt = static_cast<int>(b - a);
+}
+
 // Workspace layout (byte offsets from the caller's workspace pointer).
 struct WsLayout {
-  size_t hdr;        // uint32 err, uint32 row-item claims, uint32 column-item claims
+  size_t hdr;        // uint32 err
   size_t counts;     // uint32 [n_units]  row-statistics arrivals per unit
-  size_t done;       // uint32 [n_units]  1 once the unit's normalisers are written
   size_t beta;       // uint64 [n_units][kMaxRows]  (log2 softmax normaliser, ready tag)
   size_t clear_end;  // bytes from 0 cleared before each score call
   size_t partial;    // float2 [n_items][kMaxRows]  per-item (max, sum) in log2 units
@@ -88,13 +102,11 @@ struct ScoreParams {
   float alpha;               // log2(e) / sqrt(d)
   uint64_t wait_limit_ns;
   int32_t fault;             // test hook: 1 = unit 0 never publishes its statistics
+  int32_t lag;               // rounds a CTA's phase-1 item trails its phase-0 item
   float* mu;
   float* sigma;
   uint32_t* err;
-  uint32_t* claim1;          // next row-statistics item
-  uint32_t* claim2;          // next column-statistics item
   uint32_t* counts;
-  uint32_t* done;
   float2* partial;
   unsigned long long* beta;   // low word: beta bits, high word: 1 once written
 };
@@ -137,7 +149,7 @@ struct kve_plan {
 namespace kve {
 // Kernel launchers (defined next to their kernels).
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                         const ScoreParams& p, int num_sms, cudaStream_t stream);
+                         const ScoreParams& p, int ctas, cudaStream_t stream);
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_gather(const kve_plan& plan, const GatherParams& p, cudaStream_t stream);
 }  // namespace kve

@@ -4,37 +4,39 @@
 // L prefix keys through a causal softmax; mu_i and sigma_i are the mean and the
 // sample standard deviation of A[., i] over the n rows.
 //
-// Work is cut into items of up to kSplitKeys keys (tiles of 128). Each item runs in
+// Work is cut into items of at most kSplitTiles tiles of 128 keys. Each item runs in
 // one of two phases on a persistent, warp-specialised CTA:
 //   phase 0 (row statistics):   D[row][key] = Q K^T on tcgen05 (rows on TMEM lanes);
 //                               each epilogue thread owns one row and keeps the
 //                               running max m and sum Z = sum 2^(alpha*l - m) of its
 //                               row; the item's (m, Z) per row are published, and
 //                               the last item of a unit to publish merges them into
-//                               beta_r = log2 of the row's softmax normaliser and
-//                               raises the unit's ready flag.
+//                               beta_r = log2 of the row's softmax normaliser.
 //   phase 1 (column statistics): D[key][row] = K Q^T (keys on TMEM lanes); each
 //                               epilogue thread owns one key, forms
 //                               A = 2^(alpha*l - beta_r) for its n rows and reduces
 //                               them to mu and sigma in registers (two passes).
-// Work is claimed from two queues, both in unit order. A CTA's producer holds one
-// claimed phase-1 item and pushes it into the CTA's pipeline only once its unit's
-// statistics are merged (a relaxed poll of the unit's done flag, overlapped with
-// the loads of the current item); until then it claims phase-0 items. Nothing
-// waits on another CTA while phase-0 work remains, so the schedule needs neither an
-// ordering argument nor co-residency, and a phase-1 item re-reads its K tiles about
-// one merge latency after they were streamed, while they are still in L2. The
-// final waits (no phase-0 work left) are bounded and a timeout is reported as
-// KVE_ETIMEOUT.
+// The schedule is static. CTA c owns items c, c + G, c + 2G, ... (G CTAs, all
+// resident: the launch is cooperative), so round j is items [jG, (j+1)G) and a
+// unit's items run side by side in one round (the host picks the items per unit so
+// that rounds hold whole units). A CTA runs the phase-0 pass of its round-j item,
+// then the phase-1 pass of its round-(j - lag) item. A unit's items span at most
+// lag - 1 rounds (the host computes lag from the geometry), so every phase-1 item
+// waits only on phase-0 work that comes earlier in every CTA's sequence: there is
+// no circular wait. Between the two passes over an item's K tiles the GPU streams
+// about one round of other tiles, far less than L2 holds, so the phase-1 pass
+// reads its tiles from L2. Every cross-CTA wait is bounded and a timeout is
+// reported as KVE_ETIMEOUT.
 //
-// Roles: warp 0 claims items and issues TMA loads; warp 1 owns TMEM and issues the
-// MMAs; warp 2 (sync) does all cross-CTA work in claim order -- it publishes the
-// row statistics of phase-0 items, merges a unit's statistics when its last item
-// arrives, and stages -beta of phase-1 items in shared memory ahead of use; warps
-// 3-10 run the epilogue in two groups of four (warp w reads TMEM lanes
-// 32*(w%4)..+31), the groups taking alternate tiles. The epilogue warps never
-// touch global synchronisation; they only compute, write shared memory and
-// arrive on mbarriers.
+// Roles: warp 0 walks the item sequence and issues TMA loads; warp 1 owns TMEM and
+// issues the MMAs; warp 2 (sync) does the cross-CTA work in sequence order -- it
+// publishes the row statistics of phase-0 items and stages -beta of phase-1 items
+// in shared memory ahead of use; when a phase-0 item is the last of its unit to
+// arrive, warp 2 hands the unit to warp 3 (merge), which folds the unit's partials
+// into beta off the sequence's critical path; warps 4-11 run the epilogue in two
+// groups of four (warp w reads TMEM lanes 32*(w%4)..+31), the groups taking
+// alternate tiles. The epilogue warps never touch global synchronisation; they only
+// compute, write shared memory and arrive on mbarriers.
 #include <cstddef>
 
 #include "kve_internal.h"
@@ -43,10 +45,16 @@
 namespace kve {
 namespace {
 
-constexpr int kThreads = 352;
+constexpr int kThreads = 384;
+// Control warps come first: a scheduler that favours older warps then serves the
+// single-thread producer and MMA issuer and the latency-bound sync and merge warps
+// ahead of the throughput-bound epilogue.
 constexpr int kSyncWarp = 2;
-constexpr int kEpiWarp0 = 3;
+constexpr int kMergeWarp = 3;
+constexpr int kEpiWarp0 = 4;
 constexpr int kEpiWarps = 8;
+constexpr int kMergeSlots = 4;
+constexpr int kMergeBatch = 20;  // partials per bulk copy (1 KB each)
 constexpr int kQBufs = 2;
 constexpr int kKStages = 4;
 constexpr int kAccBufs = 4;      // 4 x 128 TMEM columns
@@ -64,15 +72,20 @@ struct ScoreCtl {
   uint64_t item_full[kItemSlots], item_empty[kItemSlots];
   uint64_t pub_full[kItemSlots];    // epilogue -> sync warp, once per item
   uint64_t beta_full[kItemSlots];   // sync warp -> epilogue, once per item
+  uint64_t merge_full[kMergeSlots], merge_empty[kMergeSlots];   // sync warp <-> merge warp
   int64_t item_ring[kItemSlots];
+  int64_t merge_job[kMergeSlots];   // unit to merge; -1 ends the merge warp
+  uint64_t merge_bar;               // bulk copies of partials
   uint32_t tmem_base;
   volatile int abort;
   int32_t roww[kMaxRows];                            // r % W
   alignas(16) float2 comb[kItemSlots][2][kMaxRows];  // per group (m, Z) of a row item
   alignas(16) float nbeta[kItemSlots][kMaxRows];     // -beta of a column item
+  alignas(16) float2 mbuf[kMergeBatch][kMaxRows];    // partials being merged
 };
 static_assert(offsetof(ScoreCtl, nbeta) % 16 == 0, "nbeta is read with 16-byte loads");
 static_assert(offsetof(ScoreCtl, comb) % 16 == 0, "comb holds float2");
+static_assert(offsetof(ScoreCtl, mbuf) % 16 == 0, "mbuf is a bulk-copy destination");
 
 struct Claim {
   int phase;
@@ -91,12 +104,6 @@ __device__ __forceinline__ Claim decode_claim(int64_t c) {
   return k;
 }
 
-__device__ __forceinline__ int item_tiles(int L, int split) {
-  const int left = L - split * kSplitKeys;
-  const int t = (left + kTileKeys - 1) / kTileKeys;
-  return t < kSplitTiles ? t : kSplitTiles;
-}
-
 __device__ __forceinline__ void set_error(const ScoreParams& P, ScoreCtl& ctl, uint32_t code) {
   atomicOr(P.err, code);
   ctl.abort = 1;
@@ -106,7 +113,7 @@ __device__ __forceinline__ void set_error(const ScoreParams& P, ScoreCtl& ctl, u
 // warp never splits in front of a .sync.aligned instruction.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, uint64_t limit,
                                           volatile int* abort) {
-  const bool ok = mbar_wait(bar, parity, global_timer_ns() + limit, abort);
+  const bool ok = mbar_wait(bar, parity, limit, abort);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -133,7 +140,8 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
   const int W = P.g.window;
   const int lim_all = u.L - W;                 // keys <= lim_all are seen by every row
   const int lim = u.L - W + ctl.roww[row];     // last key this row sees
-  const int ntiles = item_tiles(u.L, split);
+  int tile0, ntiles;
+  item_range(u, split, &tile0, &ntiles);
   const float alpha = P.alpha;
   float m = -INFINITY, Z = 0.f;
   for (int t = 0; t < ntiles; ++t, ++ai) {
@@ -150,7 +158,7 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
-    const int key0 = split * kSplitKeys + t * kTileKeys;
+    const int key0 = (tile0 + t) * kTileKeys;
     if (key0 + kTileKeys - 1 > lim_all) {
 #pragma unroll
       for (int j = 0; j < 128; ++j)
@@ -187,6 +195,77 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- epilogue, phase 1
 
+// One half (64 rows) of a key's column: A[r] = 2^(alpha*l - beta_r) for rows
+// h0..h0+63 (rows that do not see the key -- causal -- or past n give 0), the half's
+// sum and its sum of squared deviations from the half's own mean.
+template <bool kFull>
+__device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreCtl& ctl,
+                                              const float4* nb4, uint32_t taddr, int h0, int n,
+                                              int rel, float& sum, float& m2) {
+  const int nh = kFull ? 64 : (n - h0 < 64 ? n - h0 : 64);   // rows of this half, >= 1
+  float v[64];
+  tmem_ld32(taddr + h0, v);
+  if (kFull || nh > 32) tmem_ld32(taddr + h0 + 32, v + 32);
+  tmem_wait_ld();
+  const float2 a2 = make_float2(P.alpha, P.alpha);
+#pragma unroll
+  for (int r = 0; r < 64; r += 4) {
+    const float4 b = nb4[(h0 + r) >> 2];
+    const float2 x0 = ffma2(make_float2(v[r], v[r + 1]), a2, make_float2(b.x, b.y));
+    const float2 x1 = ffma2(make_float2(v[r + 2], v[r + 3]), a2, make_float2(b.z, b.w));
+    v[r] = ex2(x0.x);
+    v[r + 1] = ex2(x0.y);
+    v[r + 2] = ex2(x1.x);
+    v[r + 3] = ex2(x1.y);
+  }
+  if (rel > 0) {
+#pragma unroll
+    for (int r = 0; r < 64; ++r)
+      if (rel > ctl.roww[h0 + r]) v[r] = 0.f;
+  }
+  if (!kFull) {
+#pragma unroll
+    for (int r = 0; r < 64; ++r)
+      if (r >= nh) v[r] = 0.f;   // rows past n (not loaded when nh <= 32)
+  }
+  float2 c0 = make_float2(0.f, 0.f), c1 = c0, c2 = c0, c3 = c0;
+#pragma unroll
+  for (int r = 0; r < 64; r += 8) {
+    c0 = fadd2(c0, make_float2(v[r], v[r + 1]));
+    c1 = fadd2(c1, make_float2(v[r + 2], v[r + 3]));
+    c2 = fadd2(c2, make_float2(v[r + 4], v[r + 5]));
+    c3 = fadd2(c3, make_float2(v[r + 6], v[r + 7]));
+  }
+  const float2 cs = fadd2(fadd2(c0, c1), fadd2(c2, c3));
+  sum = cs.x + cs.y;
+  const float mh = sum / static_cast<float>(nh);
+  if (kFull) {
+    const float2 nm = make_float2(-mh, -mh);
+    float2 q0 = make_float2(0.f, 0.f), q1 = q0, q2 = q0, q3 = q0;
+#pragma unroll
+    for (int r = 0; r < 64; r += 8) {
+      const float2 d0 = fadd2(make_float2(v[r], v[r + 1]), nm);
+      const float2 d1 = fadd2(make_float2(v[r + 2], v[r + 3]), nm);
+      const float2 d2 = fadd2(make_float2(v[r + 4], v[r + 5]), nm);
+      const float2 d3 = fadd2(make_float2(v[r + 6], v[r + 7]), nm);
+      q0 = ffma2(d0, d0, q0);
+      q1 = ffma2(d1, d1, q1);
+      q2 = ffma2(d2, d2, q2);
+      q3 = ffma2(d3, d3, q3);
+    }
+    const float2 qs = fadd2(fadd2(q0, q1), fadd2(q2, q3));
+    m2 = qs.x + qs.y;
+  } else {
+    float q = 0.f;
+#pragma unroll
+    for (int r = 0; r < 64; ++r) {
+      const float d = r < nh ? v[r] - mh : 0.f;
+      q = fmaf(d, d, q);
+    }
+    m2 = q;
+  }
+}
+
 template <bool kFull>
 __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ctl,
                                               const UnitInfo& u, int split, uint32_t slot,
@@ -196,91 +275,38 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
   const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;
   const int tl = quad * 32 + lane;         // key within the tile
   const int n = kFull ? kMaxRows : P.g.n_rows;
-  const int nch = kFull ? 4 : (n + 31) / 32;
   const int W = P.g.window;
-  const float alpha = P.alpha;
-  const int ntiles = item_tiles(u.L, split);
-  const float inv_n = 1.0f / static_cast<float>(n);
+  int tile0, ntiles;
+  item_range(u, split, &tile0, &ntiles);
   const float inv_n1 = n > 1 ? 1.0f / static_cast<float>(n - 1) : 0.f;
   const float4* nb4 = reinterpret_cast<const float4*>(ctl.nbeta[slot]);
-  const float2 a2 = make_float2(alpha, alpha);
   for (int t = 0; t < ntiles; ++t, ++ai) {
     if (static_cast<int>(ai & 1u) != grp) continue;
     const uint32_t ab = ai % kAccBufs;
     if (!warp_wait(&ctl.acc_full[ab], (ai / kAccBufs) & 1u, P.wait_limit_ns, &ctl.abort))
       return false;
     tc_fence_after();
-    float v[128];
     const uint32_t taddr = ctl.tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + ab * 128u;
-#pragma unroll
-    for (int c = 0; c < 4; ++c)
-      if (c < nch) tmem_ld32(taddr + 32u * c, v + 32 * c);
-    tmem_wait_ld();
+    const int key = (tile0 + t) * kTileKeys + tl;
+    const int rel = key - (u.L - W);          // > 0: the key is inside the window
+    // the column's rows in two halves of 64 (registers), combined by the pairwise
+    // update of the mean and the sum of squared deviations (Chan, Golub, LeVeque)
+    float s1, m21, s2 = 0.f, m22 = 0.f;
+    colstats_half<kFull>(P, ctl, nb4, taddr, 0, n, rel, s1, m21);
+    const bool two = kFull || n > 64;
+    if (two) colstats_half<kFull>(P, ctl, nb4, taddr, 64, n, rel, s2, m22);
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
-    const int key = split * kSplitKeys + t * kTileKeys + tl;
-    // A[r] = 2^(alpha*l - beta_r); rows that do not see this key (causal) get 0
-#pragma unroll
-    for (int r = 0; r < 128; r += 4) {
-      if (kFull || r < n) {
-        const float4 b = nb4[r >> 2];
-        const float2 x0 = ffma2(make_float2(v[r], v[r + 1]), a2, make_float2(b.x, b.y));
-        const float2 x1 = ffma2(make_float2(v[r + 2], v[r + 3]), a2, make_float2(b.z, b.w));
-        v[r] = ex2(x0.x);
-        v[r + 1] = ex2(x0.y);
-        v[r + 2] = ex2(x1.x);
-        v[r + 3] = ex2(x1.y);
-      }
+    const float n1 = kFull ? 64.f : static_cast<float>(n < 64 ? n : 64);
+    const float n2 = static_cast<float>(n) - n1;
+    const float mu = (s1 + s2) / static_cast<float>(n);
+    float m2 = m21 + m22;
+    if (two) {
+      const float d = s2 / n2 - s1 / n1;
+      m2 = fmaf(d * d, n1 * n2 / static_cast<float>(n), m2);
     }
-    if (key > u.L - W) {
-      const int rel = key - (u.L - W);
-#pragma unroll
-      for (int r = 0; r < 128; ++r)
-        if ((kFull || r < n) && rel > ctl.roww[r]) v[r] = 0.f;
-    }
-    float mu, sigma;
-    if (kFull) {
-      float2 a0 = make_float2(0.f, 0.f), a1 = a0, a2s = a0, a3 = a0;
-#pragma unroll
-      for (int r = 0; r < 128; r += 8) {
-        a0 = fadd2(a0, make_float2(v[r], v[r + 1]));
-        a1 = fadd2(a1, make_float2(v[r + 2], v[r + 3]));
-        a2s = fadd2(a2s, make_float2(v[r + 4], v[r + 5]));
-        a3 = fadd2(a3, make_float2(v[r + 6], v[r + 7]));
-      }
-      const float2 as = fadd2(fadd2(a0, a1), fadd2(a2s, a3));
-      mu = (as.x + as.y) * inv_n;
-      const float2 nmu = make_float2(-mu, -mu);
-      float2 q0 = make_float2(0.f, 0.f), q1 = q0, q2 = q0, q3 = q0;
-#pragma unroll
-      for (int r = 0; r < 128; r += 8) {
-        const float2 d0 = fadd2(make_float2(v[r], v[r + 1]), nmu);
-        const float2 d1 = fadd2(make_float2(v[r + 2], v[r + 3]), nmu);
-        const float2 d2 = fadd2(make_float2(v[r + 4], v[r + 5]), nmu);
-        const float2 d3 = fadd2(make_float2(v[r + 6], v[r + 7]), nmu);
-        q0 = ffma2(d0, d0, q0);
-        q1 = ffma2(d1, d1, q1);
-        q2 = ffma2(d2, d2, q2);
-        q3 = ffma2(d3, d3, q3);
-      }
-      const float2 qs = fadd2(fadd2(q0, q1), fadd2(q2, q3));
-      sigma = sqrtf((qs.x + qs.y) * inv_n1);
-    } else {
-      float a = 0.f;
-#pragma unroll
-      for (int r = 0; r < 128; ++r)
-        if (r < n) a += v[r];
-      mu = a * inv_n;
-      float q = 0.f;
-#pragma unroll
-      for (int r = 0; r < 128; ++r)
-        if (r < n) {
-          const float d = v[r] - mu;
-          q = fmaf(d, d, q);
-        }
-      sigma = sqrtf(q * inv_n1);
-    }
+    const float sigma = sqrtf(fmaxf(m2, 0.f) * inv_n1);
     if (key < u.L) {
       __stcs(&P.mu[u.mu_off + key], mu);
       __stcs(&P.sigma[u.mu_off + key], sigma);
@@ -291,8 +317,8 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- sync warp
 
-// Phase-0 item: merge the two groups' (m, Z) per row, publish them, count the item,
-// and if it is the unit's last, merge all of the unit's items into beta.
+// Phase-0 item: merge the two groups' (m, Z) per row, publish them and count the
+// item. Returns whether it was the unit's last item to arrive.
 __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ctl,
                                               const UnitInfo& u, int64_t p, uint32_t slot) {
   const int lane = threadIdx.x & 31;
@@ -318,42 +344,73 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
     const uint32_t old = atomicAdd(&P.counts[u.unit], 1u);
     last = (old == static_cast<uint32_t>(u.splits - 1));
   }
-  last = __shfl_sync(0xffffffffu, last, 0);
-  if (last) {
-    __threadfence();
-    float2 acc[4];
+  return __shfl_sync(0xffffffffu, last, 0) != 0;
+}
+
+// Merge warp: fold all of a unit's (m, Z) partials into beta_r = m + log2 Z and
+// publish each row's beta with its ready tag. The partials of a unit are contiguous
+// (1 KB per item) and come in by bulk copies of up to kMergeBatch items.
+__device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, const UnitInfo& u,
+                                           uint32_t& phase) {
+  const int lane = threadIdx.x & 31;
+  const int n = P.g.n_rows;
+  __threadfence();
+  float M[4], Z[4];   // running (max, sum) per row, log2 units
 #pragma unroll
-    for (int k = 0; k < 4; ++k) acc[k] = make_float2(-INFINITY, 0.f);
-    for (int s0 = 0; s0 < u.splits; s0 += 8) {
-      float2 pz[4][8];
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int row = lane + 32 * k;
-          pz[k][j] = (s0 + j < u.splits && row < n)
-                         ? __ldcg(&P.partial[(u.item0 + s0 + j) * kMaxRows + row])
-                         : make_float2(-INFINITY, 0.f);
-        }
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[k] = merge_mz(acc[k], pz[k][j]);
+  for (int k = 0; k < 4; ++k) {
+    M[k] = -INFINITY;
+    Z[k] = 0.f;
+  }
+  for (int s0 = 0; s0 < u.splits; s0 += kMergeBatch) {
+    const int cnt = u.splits - s0 < kMergeBatch ? u.splits - s0 : kMergeBatch;
+    if (lane == 0) {
+      // the other CTAs' partials (acquired above) and this warp's reads of the
+      // previous batch come before the copy
+      fence_proxy_async();
+      const uint32_t bytes = static_cast<uint32_t>(cnt) * kMaxRows * sizeof(float2);
+      mbar_arrive_expect_tx(&ctl.merge_bar, bytes);
+      bulk_load(&ctl.mbuf[0][0], &P.partial[(u.item0 + s0) * kMaxRows], bytes, &ctl.merge_bar);
     }
+    if (!warp_wait(&ctl.merge_bar, phase, P.wait_limit_ns, &ctl.abort)) return false;
+    phase ^= 1u;
+    // all loads first (unconditional, masked afterwards), then the max, then every
+    // partial rescaled to it: the loads and the exponentials are independent
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int row = lane + 32 * k;
-      if (row < n) {
-        // one 64-bit store: a reader sees either the cleared word or (beta, 1)
-        const float b = acc[k].x + lg2(acc[k].y);
-        const unsigned long long word =
-            (1ull << 32) | static_cast<unsigned long long>(__float_as_uint(b));
-        __stcg(&P.beta[u.unit * kMaxRows + row], word);
+      float2 e[kMergeBatch];
+#pragma unroll
+      for (int j = 0; j < kMergeBatch; ++j) {
+        const float2 x = ctl.mbuf[j][row];
+        e[j] = j < cnt ? x : make_float2(-INFINITY, 0.f);
       }
+      float mb = M[k];
+#pragma unroll
+      for (int j = 0; j < kMergeBatch; ++j) mb = fmaxf(mb, e[j].x);
+      if (row >= n || mb == -INFINITY) continue;
+      float z0 = M[k] == -INFINITY ? 0.f : Z[k] * ex2(M[k] - mb), z1 = 0.f, z2 = 0.f, z3 = 0.f;
+#pragma unroll
+      for (int j = 0; j < kMergeBatch; j += 4) {
+        z0 = fmaf(e[j].y, ex2(e[j].x - mb), z0);   // ex2(-inf) = 0 for empty partials
+        if (j + 1 < kMergeBatch) z1 = fmaf(e[j + 1].y, ex2(e[j + 1].x - mb), z1);
+        if (j + 2 < kMergeBatch) z2 = fmaf(e[j + 2].y, ex2(e[j + 2].x - mb), z2);
+        if (j + 3 < kMergeBatch) z3 = fmaf(e[j + 3].y, ex2(e[j + 3].x - mb), z3);
+      }
+      M[k] = mb;
+      Z[k] = (z0 + z1) + (z2 + z3);
     }
-    __threadfence();
     __syncwarp();
-    if (lane == 0) st_release_gpu(&P.done[u.unit], 1u);   // hint for the producers
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int row = lane + 32 * k;
+    if (row < n) {
+      // one 64-bit store: a reader sees either the cleared word or (beta, 1)
+      const float b = M[k] + lg2(Z[k]);
+      const unsigned long long word =
+          (1ull << 32) | static_cast<unsigned long long>(__float_as_uint(b));
+      __stcg(&P.beta[u.unit * kMaxRows + row], word);
+    }
   }
   return true;
 }
@@ -366,7 +423,7 @@ __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ct
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   const int r0 = 4 * lane;
-  const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
+  uint64_t t0 = 0;   // timer read on the first miss only
   const volatile uint32_t* errw = P.err;
   uint32_t ns = 32;
   unsigned long long w[4];
@@ -379,7 +436,11 @@ __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ct
     for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
     if (__all_sync(0xffffffffu, ready)) break;
     int give_up = 0;
-    if (lane == 0) give_up = (*errw != 0u || ctl.abort || global_timer_ns() > deadline) ? 1 : 0;
+    if (lane == 0) {
+      const uint64_t now = global_timer_ns();
+      if (t0 == 0) t0 = now;
+      give_up = (*errw != 0u || ctl.abort || now - t0 > P.wait_limit_ns) ? 1 : 0;
+    }
     if (__shfl_sync(0xffffffffu, give_up, 0)) return false;
     __nanosleep(ns);
     if (ns < 512) ns *= 2;
@@ -420,6 +481,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl.pub_full[i], kEpiWarps);
       mbar_init(&ctl.beta_full[i], 1);
     }
+    for (int i = 0; i < kMergeSlots; ++i) {
+      mbar_init(&ctl.merge_full[i], 1);
+      mbar_init(&ctl.merge_empty[i], 1);
+    }
+    mbar_init(&ctl.merge_bar, 1);
     ctl.abort = 0;
     fence_mbar_init();
     prefetch_tensormap(&tm_q);
@@ -438,102 +504,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       uint32_t it = 0, qi = 0, ki = 0;
-      int q_used[kQBufs] = {0, 0}, k_used[kKStages] = {0, 0, 0, 0};
-      uint32_t q_last[kQBufs] = {0, 0}, k_last[kKStages] = {0, 0, 0, 0};
+      // bit i: buffer / stage i has been loaded at least once, and the parity of its last load
+      uint32_t q_used = 0, k_used = 0, q_last = 0, k_last = 0;
       const uint64_t pol_keep = l2_policy_evict_last();
       const uint64_t pol_drop = l2_policy_evict_first();
       bool ok = true;
-      // Row items are claimed one ahead. Column items are claimed only when the unit
-      // at the head of the column queue is ready: the head index and its unit's done
-      // flag are polled with relaxed loads whose values are used one item later. A
-      // claim that raced past the ready front is held until its unit is ready.
-      const volatile uint32_t* errw = P.err;
-      int s2;
-      int64_t p1 = atomicAdd(P.claim1, 1u);
-      int64_t held = -1;                               // claimed, not yet ready
-      int64_t head = 0;                                // queue head the flag refers to
-      uint32_t head_ready = 0;                         // done flag of head's unit
-      int64_t peek = 0;                                // newest peek of the queue head
-      uint32_t held_ready = 0;
+      // Own items p_j = c + j*G. Sequence: phase 0 of p_j while j - jc <= lag, else
+      // phase 1 of p_jc; phase 1 of p_jc therefore follows phase 0 of p_(jc+lag).
+      const int64_t G = gridDim.x;
+      const int64_t own = (n1 - blockIdx.x + G - 1) / G;
+      int64_t jr = 0, jc = 0;
       for (;;) {
         Claim cl;
-        bool have = false;
+        bool have = true;
         if (ctl.abort) {
           have = false;
-        } else if (held >= 0 && held_ready) {
-          cl.phase = 1;
-          cl.p = held;
-          have = true;
-          held = -1;
-        } else if (held < 0 && head < n1 && head_ready) {
-          const int64_t q = atomicAdd(P.claim2, 1u);
-          if (q < n1) {
-            if (item_unit(P.g, q, &s2) == item_unit(P.g, head, &s2)) {
-              cl.phase = 1;
-              cl.p = q;
-              have = true;
-            } else {
-              held = q;
-              held_ready = 0;
-            }
-          }
-        }
-        if (!have && !ctl.abort && p1 < n1) {
+        } else if (jr < own && jr - jc <= P.lag) {
           cl.phase = 0;
-          cl.p = p1;
-          have = true;
-          p1 = atomicAdd(P.claim1, 1u);
-        }
-        if (!have && !ctl.abort) {
-          // no row work left: wait (bounded) for column work to become ready
-          const int64_t h = ld_volatile_u32(P.claim2);
-          if (held < 0 && h >= n1) {
-            have = false;                              // all work is claimed: finish
-          } else {
-            const uint64_t deadline = global_timer_ns() + P.wait_limit_ns;
-            uint32_t ns = 64;
-            bool ready = false;
-            for (;;) {
-              const int64_t x = held >= 0 ? held : static_cast<int64_t>(ld_volatile_u32(P.claim2));
-              if (x >= n1) break;
-              if (ld_volatile_u32(&P.done[item_unit(P.g, x, &s2)])) {
-                ready = true;
-                break;
-              }
-              if (*errw != 0u || ctl.abort || global_timer_ns() > deadline) break;
-              __nanosleep(ns);
-              if (ns < 1024) ns *= 2;
-            }
-            if (held >= 0) {
-              if (!ready) {
-                ok = false;
-                break;
-              }
-              held_ready = 1;
-            } else {
-              if (!ready && ld_volatile_u32(P.claim2) < n1) {
-                ok = false;
-                break;
-              }
-              head = ld_volatile_u32(P.claim2);
-              peek = head;
-              head_ready = ready ? 1u : 0u;
-            }
-            continue;
-          }
-        }
-        // refresh the polls, consumed at the next decision: the done flag of the
-        // head peeked last time, and an independent new peek of the head
-        if (held >= 0) {
-          held_ready = ld_volatile_u32(&P.done[item_unit(P.g, held, &s2)]);
+          cl.p = blockIdx.x + jr * G;
+          ++jr;
+        } else if (jc < own) {
+          cl.phase = 1;
+          cl.p = blockIdx.x + jc * G;
+          ++jc;
         } else {
-          head = peek;
-          head_ready = head < n1 ? ld_volatile_u32(&P.done[item_unit(P.g, head, &s2)]) : 0u;
-          peek = ld_volatile_u32(P.claim2);
+          have = false;
         }
         const uint32_t slot = it % kItemSlots;
         if (!mbar_wait(&ctl.item_empty[slot], ((it / kItemSlots) & 1u) ^ 1u,
-                       global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
+                       P.wait_limit_ns, &ctl.abort)) {
           ok = false;
           break;
         }
@@ -545,7 +544,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
         const uint32_t qb = qi % kQBufs;
         if (!mbar_wait(&ctl.q_empty[qb], ((qi / kQBufs) & 1u) ^ 1u,
-                       global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
+                       P.wait_limit_ns, &ctl.abort)) {
           ok = false;
           break;
         }
@@ -553,24 +552,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d(qbuf + qb * kTileBytes, &tm_q, 0, static_cast<int32_t>(u.q_row0), &ctl.q_full[qb]);
         tma_load_2d(qbuf + qb * kTileBytes + kHalfBytes, &tm_q, 64, static_cast<int32_t>(u.q_row0),
                     &ctl.q_full[qb]);
-        q_used[qb] = 1;
-        q_last[qb] = (qi / kQBufs) & 1u;
+        q_used |= 1u << qb;
+        q_last = (q_last & ~(1u << qb)) | (((qi / kQBufs) & 1u) << qb);
         ++qi;
-        const int ntiles = item_tiles(u.L, split);
+        int tile0, ntiles;
+        item_range(u, split, &tile0, &ntiles);
         const uint64_t pol = cl.phase == 0 ? pol_keep : pol_drop;
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t ks = ki % kKStages;
           if (!mbar_wait(&ctl.k_empty[ks], ((ki / kKStages) & 1u) ^ 1u,
-                         global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
+                         P.wait_limit_ns, &ctl.abort)) {
             ok = false;
             break;
           }
-          const int32_t y = static_cast<int32_t>(u.k_row0 + split * kSplitKeys + t * kTileKeys);
+          const int32_t y = static_cast<int32_t>(u.k_row0 + (tile0 + t) * kTileKeys);
           mbar_arrive_expect_tx(&ctl.k_full[ks], kTileBytes);
           tma_load_2d_hint(kbuf + ks * kTileBytes, &tm_k, 0, y, &ctl.k_full[ks], pol);
           tma_load_2d_hint(kbuf + ks * kTileBytes + kHalfBytes, &tm_k, 64, y, &ctl.k_full[ks], pol);
-          k_used[ks] = 1;
-          k_last[ks] = (ki / kKStages) & 1u;
+          k_used |= 1u << ks;
+          k_last = (k_last & ~(1u << ks)) | (((ki / kKStages) & 1u) << ks);
           ++ki;
         }
         if (!ok) break;
@@ -579,9 +579,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // no bulk copy may still be writing shared memory when the CTA exits
       volatile int no_abort = 0;
       for (int i = 0; i < kQBufs; ++i)
-        if (q_used[i]) mbar_wait(&ctl.q_full[i], q_last[i], global_timer_ns() + P.wait_limit_ns, &no_abort);
+        if ((q_used >> i) & 1u) mbar_wait(&ctl.q_full[i], (q_last >> i) & 1u, P.wait_limit_ns, &no_abort);
       for (int i = 0; i < kKStages; ++i)
-        if (k_used[i]) mbar_wait(&ctl.k_full[i], k_last[i], global_timer_ns() + P.wait_limit_ns, &no_abort);
+        if ((k_used >> i) & 1u) mbar_wait(&ctl.k_full[i], (k_last >> i) & 1u, P.wait_limit_ns, &no_abort);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -595,7 +595,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (;;) {
         const uint32_t slot = it % kItemSlots;
         if (!mbar_wait(&ctl.item_full[slot], (it / kItemSlots) & 1u,
-                       global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
+                       P.wait_limit_ns, &ctl.abort)) {
           ok = false;
           break;
         }
@@ -607,34 +607,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         int split;
         const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
         const uint32_t qb = qi % kQBufs;
-        if (!mbar_wait(&ctl.q_full[qb], (qi / kQBufs) & 1u, global_timer_ns() + P.wait_limit_ns,
+        if (!mbar_wait(&ctl.q_full[qb], (qi / kQBufs) & 1u, P.wait_limit_ns,
                        &ctl.abort)) {
           ok = false;
           break;
         }
         ++qi;
-        const int ntiles = item_tiles(u.L, split);
+        int tile0, ntiles;
+        item_range(u, split, &tile0, &ntiles);
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t ks = ki % kKStages;
           const uint32_t ab = ai % kAccBufs;
-          if (!mbar_wait(&ctl.k_full[ks], (ki / kKStages) & 1u, global_timer_ns() + P.wait_limit_ns,
+          if (!mbar_wait(&ctl.k_full[ks], (ki / kKStages) & 1u, P.wait_limit_ns,
                          &ctl.abort) ||
               !mbar_wait(&ctl.acc_empty[ab], ((ai / kAccBufs) & 1u) ^ 1u,
-                         global_timer_ns() + P.wait_limit_ns, &ctl.abort)) {
+                         P.wait_limit_ns, &ctl.abort)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t d_tmem = ctl.tmem_base + ab * 128u;
+          // operand roles per phase are chosen once per tile: the issue loop below is
+          // branch-free (a single thread issues, so every extra instruction costs MMA rate)
+          const uint32_t qs = qaddr + qb * kTileBytes, kss = kaddr + ks * kTileBytes;
+          const uint64_t ad = sw128_desc(cl.phase == 0 ? qs : kss);
+          const uint64_t bd = sw128_desc(cl.phase == 0 ? kss : qs);
 #pragma unroll
           for (int j = 0; j < kHeadDim / 16; ++j) {
-            const uint32_t off = (j >> 2) * kHalfBytes + (j & 3) * 32u;
-            const uint64_t qd = sw128_desc(qaddr + qb * kTileBytes + off);
-            const uint64_t kd = sw128_desc(kaddr + ks * kTileBytes + off);
-            if (cl.phase == 0)
-              tc_mma_bf16(d_tmem, qd, kd, kIdesc, j > 0 ? 1u : 0u);
-            else
-              tc_mma_bf16(d_tmem, kd, qd, kIdesc, j > 0 ? 1u : 0u);
+            // the descriptor's start-address field counts 16-byte units
+            const uint64_t off = ((j >> 2) * kHalfBytes + (j & 3) * 32u) >> 4;
+            tc_mma_bf16(d_tmem, ad + off, bd + off, kIdesc, j > 0 ? 1u : 0u);
           }
           tc_commit(&ctl.k_empty[ks]);
           tc_commit(&ctl.acc_full[ab]);
@@ -651,11 +653,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       // the MMAs must have finished before TMEM is released
       volatile int no_abort = 0;
       if (issued)
-        mbar_wait(&ctl.acc_full[last_ab], last_par, global_timer_ns() + P.wait_limit_ns, &no_abort);
+        mbar_wait(&ctl.acc_full[last_ab], last_par, P.wait_limit_ns, &no_abort);
     }
   } else if (warp == kSyncWarp) {
     // ------------------------------------------------------------ sync warp
-    uint32_t it = 0;
+    uint32_t it = 0, mj = 0;
+    // hand a unit (or -1: no more units) to the merge warp
+    auto post_merge = [&](int64_t unit) -> bool {
+      const uint32_t ms = mj % kMergeSlots;
+      if (!warp_wait(&ctl.merge_empty[ms], ((mj / kMergeSlots) & 1u) ^ 1u, P.wait_limit_ns, &ctl.abort))
+        return false;
+      if (lane == 0) {
+        ctl.merge_job[ms] = unit;
+        mbar_arrive(&ctl.merge_full[ms]);
+      }
+      ++mj;
+      return true;
+    };
     for (;;) {
       const uint32_t slot = it % kItemSlots;
       const uint32_t par = (it / kItemSlots) & 1u;
@@ -664,15 +678,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       const int64_t c = ctl.item_ring[slot];
-      if (c < 0) break;
+      if (c < 0) {
+        if (!post_merge(-1)) set_error(P, ctl, 1u);
+        break;
+      }
       const Claim cl = decode_claim(c);
       int split;
       const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
       bool ok;
       if (cl.phase == 0) {
         if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);      // nothing to stage
-        ok = warp_wait(&ctl.pub_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
-             sync_rowstats(P, ctl, u, cl.p, slot);            // hands the slot back early
+        ok = warp_wait(&ctl.pub_full[slot], par, P.wait_limit_ns, &ctl.abort);
+        if (ok && sync_rowstats(P, ctl, u, cl.p, slot))       // hands the slot back early
+          ok = post_merge(u.unit);
       } else {
         ok = sync_colstats(P, ctl, u, slot);
         __syncwarp();
@@ -686,6 +704,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       ++it;
+    }
+  } else if (warp == kMergeWarp) {
+    // ------------------------------------------------------------ merge warp
+    uint32_t mj = 0, mphase = 0;
+    for (;;) {
+      const uint32_t ms = mj % kMergeSlots;
+      if (!warp_wait(&ctl.merge_full[ms], (mj / kMergeSlots) & 1u, P.wait_limit_ns, &ctl.abort)) {
+        set_error(P, ctl, 1u);
+        break;
+      }
+      const int64_t unit = ctl.merge_job[ms];
+      if (unit < 0) break;
+      if (!merge_unit(P, ctl, unit_info(P.g, unit), mphase)) {
+        set_error(P, ctl, 1u);
+        // no bulk copy may still be writing shared memory when the CTA exits
+        volatile int no_abort = 0;
+        if (lane == 0) mbar_wait(&ctl.merge_bar, mphase, P.wait_limit_ns, &no_abort);
+        break;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.merge_empty[ms]);
+      ++mj;
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -733,16 +773,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                         const ScoreParams& p, int num_sms, cudaStream_t stream) {
+                         const ScoreParams& p, int ctas, cudaStream_t stream) {
   const bool full = plan.geo.n_rows == kMaxRows;
   auto* fn = full ? score_kernel<true> : score_kernel<false>;
   cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kDynSmem));
   if (e != cudaSuccess) return e;
-  const int64_t items = p.g.n_items;
-  const int grid = static_cast<int>(items < num_sms ? items : num_sms);
-  fn<<<grid, kThreads, kDynSmem, stream>>>(tm_q, tm_k, p);
-  return cudaGetLastError();
+  // CTAs wait on each other's row statistics: all of them must be resident at once
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ctas));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kDynSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, fn, tm_q, tm_k, p);
 }
 
 }  // namespace kve
