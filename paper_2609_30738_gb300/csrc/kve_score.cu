@@ -415,26 +415,40 @@ __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, 
   return true;
 }
 
-// Phase-1 item: wait for the unit's merged statistics and stage -beta. Each row's
-// normaliser carries its own ready tag, so one round of loads both checks and
-// fetches it.
-__device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, uint32_t slot) {
+// Phase-1 item: one round of loads of the unit's normalisers. Each row's word carries
+// its own ready tag; when every row is ready, -beta is staged in shared memory for
+// the epilogue and true is returned.
+__device__ __forceinline__ bool try_stage_beta(const ScoreParams& P, ScoreCtl& ctl, int64_t unit,
+                                               uint32_t slot) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   const int r0 = 4 * lane;
+  unsigned long long w[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    w[k] = (r0 + k < n) ? __ldcg(&P.beta[unit * kMaxRows + r0 + k]) : (1ull << 32);
+  bool ready = true;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
+  if (!__all_sync(0xffffffffu, ready)) return false;
+  float4 b;
+  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
+  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
+  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
+  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
+  reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
+  return true;
+}
+
+// Phase-1 item: wait (bounded) for the unit's merged statistics and stage -beta.
+__device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ctl, int64_t unit,
+                                              uint32_t slot) {
+  const int lane = threadIdx.x & 31;
   uint64_t t0 = 0;   // timer read on the first miss only
   const volatile uint32_t* errw = P.err;
   uint32_t ns = 32;
-  unsigned long long w[4];
   for (;;) {
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-      w[k] = (r0 + k < n) ? __ldcg(&P.beta[u.unit * kMaxRows + r0 + k]) : (1ull << 32);
-    bool ready = true;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
-    if (__all_sync(0xffffffffu, ready)) break;
+    if (try_stage_beta(P, ctl, unit, slot)) return true;
     int give_up = 0;
     if (lane == 0) {
       const uint64_t now = global_timer_ns();
@@ -445,13 +459,6 @@ __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ct
     __nanosleep(ns);
     if (ns < 512) ns *= 2;
   }
-  float4 b;
-  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
-  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
-  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
-  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
-  reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
-  return true;
 }
 
 // ---------------------------------------------------------------- kernel
@@ -670,7 +677,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++mj;
       return true;
     };
+    bool staged = false;   // item `it` is a phase-1 item already staged and released
     for (;;) {
+      if (staged) {
+        // its slot may already hold a later item: never wait on it again
+        staged = false;
+        ++it;
+        continue;
+      }
       const uint32_t slot = it % kItemSlots;
       const uint32_t par = (it / kItemSlots) & 1u;
       if (!warp_wait(&ctl.item_full[slot], par, P.wait_limit_ns, &ctl.abort)) {
@@ -685,14 +699,51 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Claim cl = decode_claim(c);
       int split;
       const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
-      bool ok;
+      bool ok = true;
+      bool next_staged = false;
       if (cl.phase == 0) {
         if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);      // nothing to stage
-        ok = warp_wait(&ctl.pub_full[slot], par, P.wait_limit_ns, &ctl.abort);
+        // While the epilogue finishes this item, stage the next item's normalisers
+        // if it is a phase-1 item whose unit is already merged.
+        const uint32_t nslot = (it + 1) % kItemSlots;
+        const uint32_t npar = ((it + 1) / kItemSlots) & 1u;
+        bool next_checked = false;
+        uint64_t t0 = 0;
+        for (;;) {
+          if (__all_sync(0xffffffffu, mbar_try_wait(&ctl.pub_full[slot], par))) break;
+          if (!next_checked && __all_sync(0xffffffffu, mbar_try_wait(&ctl.item_full[nslot], npar))) {
+            const int64_t cn = ctl.item_ring[nslot];
+            if (cn < 0 || decode_claim(cn).phase == 0) {
+              next_checked = true;
+            } else {
+              int sn;
+              const int64_t un = item_unit(P.g, decode_claim(cn).p, &sn);
+              if (try_stage_beta(P, ctl, un, nslot)) {
+                // the sync warp's whole part in that item is done: release it now
+                next_checked = next_staged = true;
+                __syncwarp();
+                if (lane == 0) {
+                  mbar_arrive(&ctl.beta_full[nslot]);
+                  mbar_arrive(&ctl.item_empty[nslot]);
+                }
+              }
+            }
+          }
+          int give_up = 0;
+          if (lane == 0) {
+            const uint64_t now = global_timer_ns();
+            if (t0 == 0) t0 = now;
+            give_up = (ctl.abort || now - t0 > P.wait_limit_ns) ? 1 : 0;
+          }
+          if (__shfl_sync(0xffffffffu, give_up, 0)) {
+            ok = false;
+            break;
+          }
+        }
         if (ok && sync_rowstats(P, ctl, u, cl.p, slot))       // hands the slot back early
           ok = post_merge(u.unit);
       } else {
-        ok = sync_colstats(P, ctl, u, slot);
+        ok = sync_colstats(P, ctl, u.unit, slot);
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&ctl.beta_full[slot]);
@@ -703,6 +754,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         set_error(P, ctl, 1u);
         break;
       }
+      staged = next_staged;
       ++it;
     }
   } else if (warp == kMergeWarp) {
