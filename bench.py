@@ -38,7 +38,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one score-kernel launch (dram__bytes_read.sum + dram__bytes_write.sum),
 # from the ncu capture summarised in profiles/, valid only for the kernel source it was
 # taken on (sha256 of csrc/kve_score.cu); per launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": None, "bytes_per_launch": None}
+SCORE_TRAFFIC = {"source_sha256": "a45fbc449a0b2500067bec12e0d46ba9207ff22ceb6f33680a9c40770aca38ea",
+                 "bytes_per_launch": 2176911104 + 74189312}
 
 
 def _score_source_sha():
