@@ -164,10 +164,17 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
       for (int j = 0; j < 128; ++j)
         if (key0 + j > lim) v[j] = -INFINITY;
     }
-    float mx = v[0];
+    float q0 = v[0], q1 = v[1], q2 = v[2], q3 = v[3];
 #pragma unroll
-    for (int j = 1; j + 1 < 128; j += 2) mx = max3(mx, v[j], v[j + 1]);
-    mx = fmaxf(mx, v[127]);
+    for (int j = 4; j < 124; j += 8) {
+      q0 = max3(q0, v[j], v[j + 1]);
+      q1 = max3(q1, v[j + 2], v[j + 3]);
+      q2 = max3(q2, v[j + 4], v[j + 5]);
+      q3 = max3(q3, v[j + 6], v[j + 7]);
+    }
+    q0 = max3(q0, v[124], v[125]);
+    q1 = max3(q1, v[126], v[127]);
+    const float mx = fmaxf(fmaxf(q0, q1), fmaxf(q2, q3));
     const float mn = fmaxf(m, mx * alpha);
     if (mn != -INFINITY) {
       const float2 a2 = make_float2(alpha, alpha);
@@ -291,10 +298,15 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     const int rel = key - (u.L - W);          // > 0: the key is inside the window
     // the column's rows in two halves of 64 (registers), combined by the pairwise
     // update of the mean and the sum of squared deviations (Chan, Golub, LeVeque)
-    float s1, m21, s2 = 0.f, m22 = 0.f;
-    colstats_half<kFull>(P, ctl, nb4, taddr, 0, n, rel, s1, m21);
+    float hs[2] = {0.f, 0.f}, hm2[2] = {0.f, 0.f};
     const bool two = kFull || n > 64;
-    if (two) colstats_half<kFull>(P, ctl, nb4, taddr, 64, n, rel, s2, m22);
+#pragma unroll 1
+    for (int h = 0; h < (two ? 2 : 1); ++h) {
+      float sh, mh2;
+      colstats_half<kFull>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, mh2);
+      if (h == 0) { hs[0] = sh; hm2[0] = mh2; } else { hs[1] = sh; hm2[1] = mh2; }
+    }
+    const float s1 = hs[0], m21 = hm2[0], s2 = hs[1], m22 = hm2[1];
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
