@@ -65,6 +65,33 @@ constexpr uint32_t kTmemCols = 512;
 constexpr size_t kDynSmem = (kQBufs + kKStages) * kTileBytes + 1024;
 constexpr uint32_t kIdesc = idesc_bf16_f32(128, 128);
 
+// One pass over one item, as the producer derives it once from the item index and
+// hands it to the other roles through the item ring (p = -1 ends the work).
+struct ItemDesc {
+  int64_t p;         // item index
+  int64_t unit;
+  int64_t mu_off;    // first mu/sigma element of the unit
+  int64_t item0;     // first item of the unit
+  int32_t phase;     // 0: row statistics, 1: column statistics
+  int32_t tile0;     // first tile of the item within the unit
+  int32_t ntiles;
+  int32_t L;         // prefix length of the unit
+  int32_t splits;    // items of the unit
+  int32_t pad;
+};
+
+struct Claim {
+  int phase;
+  int64_t p;
+};
+
+struct MergeJob {
+  int64_t unit;      // -1: no more units
+  int64_t item0;
+  int32_t splits;
+  int32_t pad;
+};
+
 struct ScoreCtl {
   uint64_t q_full[kQBufs], q_empty[kQBufs];
   uint64_t k_full[kKStages], k_empty[kKStages];
@@ -73,8 +100,8 @@ struct ScoreCtl {
   uint64_t pub_full[kItemSlots];    // epilogue -> sync warp, once per item
   uint64_t beta_full[kItemSlots];   // sync warp -> epilogue, once per item
   uint64_t merge_full[kMergeSlots], merge_empty[kMergeSlots];   // sync warp <-> merge warp
-  int64_t item_ring[kItemSlots];
-  int64_t merge_job[kMergeSlots];   // unit to merge; -1 ends the merge warp
+  ItemDesc item_ring[kItemSlots];   // written by the producer, read by every role
+  MergeJob merge_job[kMergeSlots];  // unit to merge; unit -1 ends the merge warp
   uint64_t merge_bar;               // bulk copies of partials
   uint32_t tmem_base;
   volatile int abort;
@@ -87,22 +114,6 @@ static_assert(offsetof(ScoreCtl, nbeta) % 16 == 0, "nbeta is read with 16-byte l
 static_assert(offsetof(ScoreCtl, comb) % 16 == 0, "comb holds float2");
 static_assert(offsetof(ScoreCtl, mbuf) % 16 == 0, "mbuf is a bulk-copy destination");
 
-struct Claim {
-  int phase;
-  int64_t p;
-};
-
-// Ring entry: item index in the low bits, phase in bit 62; -1 ends the work.
-__device__ __forceinline__ int64_t encode_claim(int phase, int64_t p) {
-  return p | (static_cast<int64_t>(phase) << 62);
-}
-
-__device__ __forceinline__ Claim decode_claim(int64_t c) {
-  Claim k;
-  k.phase = static_cast<int>((c >> 62) & 1);
-  k.p = c & ((int64_t(1) << 62) - 1);
-  return k;
-}
 
 __device__ __forceinline__ void set_error(const ScoreParams& P, ScoreCtl& ctl, uint32_t code) {
   atomicOr(P.err, code);
@@ -131,17 +142,15 @@ __device__ __forceinline__ float2 merge_mz(float2 a, float2 b) {
 
 template <bool kFull>
 __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, int split, uint32_t slot,
-                                              uint32_t& ai) {
+                                              const ItemDesc& d, uint32_t slot, uint32_t& ai) {
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
   const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;   // 0 or 1
   const int row = quad * 32 + lane;
   const int W = P.g.window;
-  const int lim_all = u.L - W;                 // keys <= lim_all are seen by every row
-  const int lim = u.L - W + ctl.roww[row];     // last key this row sees
-  int tile0, ntiles;
-  item_range(u, split, &tile0, &ntiles);
+  const int lim_all = d.L - W;                 // keys <= lim_all are seen by every row
+  const int lim = d.L - W + ctl.roww[row];     // last key this row sees
+  const int tile0 = d.tile0, ntiles = d.ntiles;
   const float alpha = P.alpha;
   float m = -INFINITY, Z = 0.f;
   for (int t = 0; t < ntiles; ++t, ++ai) {
@@ -275,16 +284,14 @@ __device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreC
 
 template <bool kFull>
 __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, int split, uint32_t slot,
-                                              uint32_t& ai) {
+                                              const ItemDesc& d, uint32_t slot, uint32_t& ai) {
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
   const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;
   const int tl = quad * 32 + lane;         // key within the tile
   const int n = kFull ? kMaxRows : P.g.n_rows;
   const int W = P.g.window;
-  int tile0, ntiles;
-  item_range(u, split, &tile0, &ntiles);
+  const int tile0 = d.tile0, ntiles = d.ntiles;
   const float inv_n1 = n > 1 ? 1.0f / static_cast<float>(n - 1) : 0.f;
   const float4* nb4 = reinterpret_cast<const float4*>(ctl.nbeta[slot]);
   for (int t = 0; t < ntiles; ++t, ++ai) {
@@ -295,7 +302,7 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     tc_fence_after();
     const uint32_t taddr = ctl.tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + ab * 128u;
     const int key = (tile0 + t) * kTileKeys + tl;
-    const int rel = key - (u.L - W);          // > 0: the key is inside the window
+    const int rel = key - (d.L - W);          // > 0: the key is inside the window
     // the column's rows in two halves of 64 (registers), combined by the pairwise
     // update of the mean and the sum of squared deviations (Chan, Golub, LeVeque)
     float hs[2] = {0.f, 0.f}, hm2[2] = {0.f, 0.f};
@@ -319,9 +326,9 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
       m2 = fmaf(d * d, n1 * n2 / static_cast<float>(n), m2);
     }
     const float sigma = sqrtf(fmaxf(m2, 0.f) * inv_n1);
-    if (key < u.L) {
-      __stcs(&P.mu[u.mu_off + key], mu);
-      __stcs(&P.sigma[u.mu_off + key], sigma);
+    if (key < d.L) {
+      __stcs(&P.mu[d.mu_off + key], mu);
+      __stcs(&P.sigma[d.mu_off + key], sigma);
     }
   }
   return true;
@@ -332,7 +339,7 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
 // Phase-0 item: merge the two groups' (m, Z) per row, publish them and count the
 // item. Returns whether it was the unit's last item to arrive.
 __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ctl,
-                                              const UnitInfo& u, int64_t p, uint32_t slot) {
+                                              const ItemDesc& d, uint32_t slot) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   float2 mz[4];
@@ -347,14 +354,14 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const int row = lane + 32 * k;
-    if (row < n) P.partial[p * kMaxRows + row] = mz[k];
+    if (row < n) P.partial[d.p * kMaxRows + row] = mz[k];
   }
   __threadfence();
   __syncwarp();
   int last = 0;
-  if (lane == 0 && !(P.fault == 1 && u.unit == 0)) {
-    const uint32_t old = atomicAdd(&P.counts[u.unit], 1u);
-    last = (old == static_cast<uint32_t>(u.splits - 1));
+  if (lane == 0 && !(P.fault == 1 && d.unit == 0)) {
+    const uint32_t old = atomicAdd(&P.counts[d.unit], 1u);
+    last = (old == static_cast<uint32_t>(d.splits - 1));
   }
   return __shfl_sync(0xffffffffu, last, 0) != 0;
 }
@@ -362,7 +369,7 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
 // Merge warp: fold all of a unit's (m, Z) partials into beta_r = m + log2 Z and
 // publish each row's beta with its ready tag. The partials of a unit are contiguous
 // (1 KB per item) and come in by bulk copies of up to kMergeBatch items.
-__device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, const UnitInfo& u,
+__device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, const MergeJob& u,
                                            uint32_t& phase) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
@@ -555,12 +562,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        ctl.item_ring[slot] = have ? encode_claim(cl.phase, cl.p) : -1;
+        ItemDesc d;
+        UnitInfo u;
+        if (have) {
+          int split;
+          u = unit_info(P.g, item_unit(P.g, cl.p, &split));
+          d.p = cl.p;
+          d.unit = u.unit;
+          d.mu_off = u.mu_off;
+          d.item0 = u.item0;
+          d.phase = cl.phase;
+          item_range(u, split, &d.tile0, &d.ntiles);
+          d.L = u.L;
+          d.splits = u.splits;
+          d.pad = 0;
+        } else {
+          d.p = -1;
+        }
+        ctl.item_ring[slot] = d;
         mbar_arrive(&ctl.item_full[slot]);
         ++it;
         if (!have) break;
-        int split;
-        const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
         const uint32_t qb = qi % kQBufs;
         if (!mbar_wait(&ctl.q_empty[qb], ((qi / kQBufs) & 1u) ^ 1u,
                        P.wait_limit_ns, &ctl.abort)) {
@@ -574,8 +596,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         q_used |= 1u << qb;
         q_last = (q_last & ~(1u << qb)) | (((qi / kQBufs) & 1u) << qb);
         ++qi;
-        int tile0, ntiles;
-        item_range(u, split, &tile0, &ntiles);
+        const int tile0 = d.tile0, ntiles = d.ntiles;
         const uint64_t pol = cl.phase == 0 ? pol_keep : pol_drop;
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t ks = ki % kKStages;
@@ -618,13 +639,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        const int64_t c = ctl.item_ring[slot];
+        const int phase = ctl.item_ring[slot].phase;
+        const int ntiles = ctl.item_ring[slot].ntiles;
+        const bool end = ctl.item_ring[slot].p < 0;
         mbar_arrive(&ctl.item_empty[slot]);
         ++it;
-        if (c < 0) break;
-        const Claim cl = decode_claim(c);
-        int split;
-        const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
+        if (end) break;
         const uint32_t qb = qi % kQBufs;
         if (!mbar_wait(&ctl.q_full[qb], (qi / kQBufs) & 1u, P.wait_limit_ns,
                        &ctl.abort)) {
@@ -632,8 +652,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         ++qi;
-        int tile0, ntiles;
-        item_range(u, split, &tile0, &ntiles);
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t ks = ki % kKStages;
           const uint32_t ab = ai % kAccBufs;
@@ -649,8 +667,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           // operand roles per phase are chosen once per tile: the issue loop below is
           // branch-free (a single thread issues, so every extra instruction costs MMA rate)
           const uint32_t qs = qaddr + qb * kTileBytes, kss = kaddr + ks * kTileBytes;
-          const uint64_t ad = sw128_desc(cl.phase == 0 ? qs : kss);
-          const uint64_t bd = sw128_desc(cl.phase == 0 ? kss : qs);
+          const uint64_t ad = sw128_desc(phase == 0 ? qs : kss);
+          const uint64_t bd = sw128_desc(phase == 0 ? kss : qs);
 #pragma unroll
           for (int j = 0; j < kHeadDim / 16; ++j) {
             // the descriptor's start-address field counts 16-byte units
@@ -678,12 +696,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ sync warp
     uint32_t it = 0, mj = 0;
     // hand a unit (or -1: no more units) to the merge warp
-    auto post_merge = [&](int64_t unit) -> bool {
+    auto post_merge = [&](const MergeJob& job) -> bool {
       const uint32_t ms = mj % kMergeSlots;
       if (!warp_wait(&ctl.merge_empty[ms], ((mj / kMergeSlots) & 1u) ^ 1u, P.wait_limit_ns, &ctl.abort))
         return false;
       if (lane == 0) {
-        ctl.merge_job[ms] = unit;
+        ctl.merge_job[ms] = job;
         mbar_arrive(&ctl.merge_full[ms]);
       }
       ++mj;
@@ -703,17 +721,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         set_error(P, ctl, 1u);
         break;
       }
-      const int64_t c = ctl.item_ring[slot];
-      if (c < 0) {
-        if (!post_merge(-1)) set_error(P, ctl, 1u);
+      const ItemDesc d = ctl.item_ring[slot];
+      if (d.p < 0) {
+        MergeJob none;
+        none.unit = -1;
+        if (!post_merge(none)) set_error(P, ctl, 1u);
         break;
       }
-      const Claim cl = decode_claim(c);
-      int split;
-      const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
       bool ok = true;
       bool next_staged = false;
-      if (cl.phase == 0) {
+      if (d.phase == 0) {
         if (lane == 0) mbar_arrive(&ctl.beta_full[slot]);      // nothing to stage
         // While the epilogue finishes this item, stage the next item's normalisers
         // if it is a phase-1 item whose unit is already merged.
@@ -724,13 +741,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (;;) {
           if (__all_sync(0xffffffffu, mbar_try_wait(&ctl.pub_full[slot], par))) break;
           if (!next_checked && __all_sync(0xffffffffu, mbar_try_wait(&ctl.item_full[nslot], npar))) {
-            const int64_t cn = ctl.item_ring[nslot];
-            if (cn < 0 || decode_claim(cn).phase == 0) {
+            const int64_t pn = ctl.item_ring[nslot].p;
+            const int phn = ctl.item_ring[nslot].phase;
+            if (pn < 0 || phn == 0) {
               next_checked = true;
             } else {
-              int sn;
-              const int64_t un = item_unit(P.g, decode_claim(cn).p, &sn);
-              if (try_stage_beta(P, ctl, un, nslot)) {
+              if (try_stage_beta(P, ctl, ctl.item_ring[nslot].unit, nslot)) {
                 // the sync warp's whole part in that item is done: release it now
                 next_checked = next_staged = true;
                 __syncwarp();
@@ -752,10 +768,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
         }
-        if (ok && sync_rowstats(P, ctl, u, cl.p, slot))       // hands the slot back early
-          ok = post_merge(u.unit);
+        if (ok && sync_rowstats(P, ctl, d, slot)) {           // hands the slot back early
+          MergeJob job;
+          job.unit = d.unit;
+          job.item0 = d.item0;
+          job.splits = d.splits;
+          job.pad = 0;
+          ok = post_merge(job);
+        }
       } else {
-        ok = sync_colstats(P, ctl, u.unit, slot);
+        ok = sync_colstats(P, ctl, d.unit, slot);
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&ctl.beta_full[slot]);
@@ -778,9 +800,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         set_error(P, ctl, 1u);
         break;
       }
-      const int64_t unit = ctl.merge_job[ms];
-      if (unit < 0) break;
-      if (!merge_unit(P, ctl, unit_info(P.g, unit), mphase)) {
+      const MergeJob job = ctl.merge_job[ms];
+      if (job.unit < 0) break;
+      if (!merge_unit(P, ctl, job, mphase)) {
         set_error(P, ctl, 1u);
         // no bulk copy may still be writing shared memory when the CTA exits
         volatile int no_abort = 0;
@@ -801,17 +823,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         set_error(P, ctl, 1u);
         break;
       }
-      const int64_t c = ctl.item_ring[slot];
-      if (c < 0) break;
-      const Claim cl = decode_claim(c);
-      int split;
-      const UnitInfo u = unit_info(P.g, item_unit(P.g, cl.p, &split));
+      const ItemDesc d = ctl.item_ring[slot];
+      if (d.p < 0) break;
       bool ok;
-      if (cl.phase == 0) {
-        ok = rowstats_item<kFull>(P, ctl, u, split, slot, ai);
+      if (d.phase == 0) {
+        ok = rowstats_item<kFull>(P, ctl, d, slot, ai);
       } else {
         ok = warp_wait(&ctl.beta_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
-             colstats_item<kFull>(P, ctl, u, split, slot, ai);
+             colstats_item<kFull>(P, ctl, d, slot, ai);
       }
       if (!ok) {
         set_error(P, ctl, 1u);
