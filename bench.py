@@ -36,15 +36,18 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 
 # DRAM traffic of one score-kernel launch (dram__bytes_read.sum + dram__bytes_write.sum),
-# from the ncu capture summarised in profiles/, valid only for the kernel source it was
-# taken on (sha256 of csrc/kve_score.cu); per launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "a45fbc449a0b2500067bec12e0d46ba9207ff22ceb6f33680a9c40770aca38ea",
-                 "bytes_per_launch": 2176911104 + 74189312}
+# from the ncu capture summarised in profiles/, valid only for the sources it was taken
+# on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
+# launch of the full workload.
+SCORE_TRAFFIC = {"source_sha256": "16e5dffa8c41de8c22e969acfe5d69277e1e11c6e3dcb3ccd7e2b60a1ddbf733",
+                 "bytes_per_launch": 3499451392 + 74934272}
 
 
 def _score_source_sha():
-    p = os.path.join(ROOT, "paper_2609_30738_gb300", "csrc", "kve_score.cu")
-    return hashlib.sha256(open(p, "rb").read()).hexdigest()
+    h = hashlib.sha256()
+    for f in ("kve_score.cu", "kve_host.cu"):
+        h.update(open(os.path.join(ROOT, "paper_2609_30738_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
 
 
 def _peaks():
