@@ -28,7 +28,7 @@ constexpr int kChunks = kHeadDim / 8;   // 16-byte chunks of a key row
 constexpr int kBins = 4096;             // radix digits of the first two passes
 constexpr int kPoolRun = 7;             // consecutive pooled outputs per run (odd: the
                                         // runs of a warp start on distinct banks)
-constexpr int kPoolRuns = 4;            // runs per thread and tile
+constexpr int kPoolRuns = 2;            // runs per thread and tile
 constexpr int kBatch = 16;              // key loads in flight per thread
 constexpr int kTieCap = 2048;           // cut ties gathered in shared memory
 
@@ -131,29 +131,31 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     constexpr int kTile = NT * kPoolRun * kPoolRuns;
     const int tile_in = kTile + 2 * h;
     float* tsg = tmu + tile_in;
+    // the loads of the next tile are in flight while this tile is pooled
+    constexpr int kPer = (kTile + 2 * 127 + NT - 1) / NT;
+    float lm[kPer], ls[kPer];
+    auto load_tile = [&](int base) {
+#pragma unroll
+      for (int q = 0; q < kPer; ++q) {
+        const int j = q * NT + tid;
+        const int i = base - h + j;
+        const bool in = (j < tile_in) && (i >= 0) && (i < Lc);
+        lm[q] = in ? __ldg(mu + i) : -INFINITY;
+        ls[q] = in ? __ldg(sg + i) : -INFINITY;
+      }
+    };
+    load_tile(0);
     for (int base = 0; base < Lc; base += kTile) {
-      {
-        // every load of the tile is issued before the first store (one round trip)
-        constexpr int kPer = (kTile + 2 * 127 + NT - 1) / NT;
-        float lm[kPer], ls[kPer];
 #pragma unroll
-        for (int q = 0; q < kPer; ++q) {
-          const int j = q * NT + tid;
-          const int i = base - h + j;
-          const bool in = (j < tile_in) && (i >= 0) && (i < Lc);
-          lm[q] = in ? __ldg(mu + i) : -INFINITY;
-          ls[q] = in ? __ldg(sg + i) : -INFINITY;
-        }
-#pragma unroll
-        for (int q = 0; q < kPer; ++q) {
-          const int j = q * NT + tid;
-          if (j < tile_in) {
-            tmu[j] = lm[q];
-            tsg[j] = ls[q];
-          }
+      for (int q = 0; q < kPer; ++q) {
+        const int j = q * NT + tid;
+        if (j < tile_in) {
+          tmu[j] = lm[q];
+          tsg[j] = ls[q];
         }
       }
       __syncthreads();
+      if (base + kTile < Lc) load_tile(base + kTile);
 #pragma unroll
       for (int q = 0; q < kPoolRuns; ++q) {
         const int o0 = (q * NT + tid) * kPoolRun;
