@@ -65,6 +65,22 @@ def _dist():
     return world, rank, local
 
 
+def _max_over_ranks(x, world, device):
+    """Job time = the slowest rank's time (every rank holds the max afterwards)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _job_tok_s(world, prefix_len, step_s):
+    """Whole-job throughput: every rank evicts one request of prefix_len tokens per step."""
+    return world * prefix_len / step_s
+
+
 class ClockSampler:
     """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
 
@@ -309,10 +325,7 @@ def run_ours(args):
     clocks = sampler.stop() if sampler else None
     if plan.status(bufs.ws, stream) != K.KVE_OK:
         raise RuntimeError("device-side wait timed out in the timed region")
-    if world > 1:
-        t = torch.tensor([elapsed], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed = float(t.item())
+    elapsed = _max_over_ranks(elapsed, world, dev)
 
     # end to end through the public API with host buffers (pinned), copies inside
     e2e = None
@@ -348,13 +361,10 @@ def run_ours(args):
         b.record(stream)
         torch.cuda.synchronize()
         e2e_s = a.elapsed_time(b) / 1e3 / args.e2e_steps
-        if world > 1:
-            t = torch.tensor([e2e_s], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t.item())
+        e2e_s = _max_over_ranks(e2e_s, world, dev)
         h2d = sum(x.numel() * x.element_size() for x in (hq, hk, hv))
         d2h = sum(x.numel() * x.element_size() for x in (o_idx, o_k, o_v))
-        e2e = {"value": world * L / e2e_s, "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": _job_tok_s(world, L, e2e_s), "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3}
         del hq, hk, hv, dq, dk, dv
 
@@ -377,7 +387,7 @@ def run_ours(args):
         cpu = cpu_baseline_from_device(spec, batch, args.cpu_units)
 
     step_s = elapsed / args.steps
-    line = {"metric": METRIC, "value": world * L / step_s, "unit": "prefix tok/s", "n_gpus": world,
+    line = {"metric": METRIC, "value": _job_tok_s(world, L, step_s), "unit": "prefix tok/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16xbf16->f32", "data": "synthetic (seeded Mistral-7B-shaped K/V/Q)",
