@@ -39,8 +39,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "16e5dffa8c41de8c22e969acfe5d69277e1e11c6e3dcb3ccd7e2b60a1ddbf733",
-                 "bytes_per_launch": 3499451392 + 74934272}
+SCORE_TRAFFIC = {"source_sha256": "51b6660f9826d925d6e9327ed1c279162e393d3cca5c1ea293644a0b70007755",
+                 "bytes_per_launch": 2178510080 + 74864128}
 
 
 def _score_source_sha():

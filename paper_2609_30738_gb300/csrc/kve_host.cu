@@ -74,11 +74,11 @@ int32_t choose_splits(int64_t T, int64_t ctas) {
   return static_cast<int32_t>(kmin);
 }
 
-// Rounds a CTA's phase-1 item trails its phase-0 item in the score kernel. Any lag
-// at least the number of rounds a unit's items span is free of circular waits; two
-// rounds more than that span give a unit's merge (about half a round) time to land
-// before its first phase-1 item comes up, while the K tiles of the rounds in between
-// (about 3 x 32 MB at full width) still fit in L2.
+// Rounds a CTA's phase-1 item trails its phase-0 item in the score kernel: one more
+// than the most rounds any unit's items span. Any lag at least that span is free of
+// circular waits; the extra round gives a unit's merge time to land before its first
+// phase-1 item, while the K tiles streamed in between (two rounds, about 64 MB at full
+// width) stay in L2 for the phase-1 re-read.
 int32_t score_lag(const kve::Geometry& g, int64_t ctas) {
   int64_t span = 0;
   const int64_t units_per_req = static_cast<int64_t>(g.num_layers) * g.hkv;
@@ -91,7 +91,7 @@ int32_t score_lag(const kve::Geometry& g, int64_t ctas) {
       span = std::max<int64_t>(span, (a + k - 1) / ctas - a / ctas);
     }
   }
-  return static_cast<int32_t>(span + 2);
+  return static_cast<int32_t>(span + 1);
 }
 
 }  // namespace

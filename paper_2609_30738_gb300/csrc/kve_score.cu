@@ -54,15 +54,16 @@ constexpr int kMergeWarp = 3;
 constexpr int kEpiWarp0 = 4;
 constexpr int kEpiWarps = 8;
 constexpr int kMergeSlots = 4;
-constexpr int kMergeBatch = 20;  // partials per bulk copy (1 KB each)
+constexpr int kMergeBatch = 40;  // partials per bulk copy (1 KB each): a 38-item unit in one
 constexpr int kQBufs = 2;
-constexpr int kKStages = 4;
+constexpr int kKStages = 3;      // K tiles in flight (32 KB each)
 constexpr int kAccBufs = 4;      // 4 x 128 TMEM columns
 constexpr int kItemSlots = 4;
 constexpr uint32_t kTileBytes = 128 * kHeadDim * 2;   // 32 KB: 128 rows x 128 bf16
 constexpr uint32_t kHalfBytes = kTileBytes / 2;       // one 64-element (128 B) column block
 constexpr uint32_t kTmemCols = 512;
-constexpr size_t kDynSmem = (kQBufs + kKStages) * kTileBytes + 1024;
+constexpr size_t kMergeBytes = static_cast<size_t>(kMergeBatch) * kMaxRows * sizeof(float2);
+constexpr size_t kDynSmem = (kQBufs + kKStages) * kTileBytes + kMergeBytes + 1024;
 constexpr uint32_t kIdesc = idesc_bf16_f32(128, 128);
 
 // One pass over one item, as the producer derives it once from the item index and
@@ -108,11 +109,9 @@ struct ScoreCtl {
   int32_t roww[kMaxRows];                            // r % W
   alignas(16) float2 comb[kItemSlots][2][kMaxRows];  // per group (m, Z) of a row item
   alignas(16) float nbeta[kItemSlots][kMaxRows];     // -beta of a column item
-  alignas(16) float2 mbuf[kMergeBatch][kMaxRows];    // partials being merged
 };
 static_assert(offsetof(ScoreCtl, nbeta) % 16 == 0, "nbeta is read with 16-byte loads");
 static_assert(offsetof(ScoreCtl, comb) % 16 == 0, "comb holds float2");
-static_assert(offsetof(ScoreCtl, mbuf) % 16 == 0, "mbuf is a bulk-copy destination");
 
 
 __device__ __forceinline__ void set_error(const ScoreParams& P, ScoreCtl& ctl, uint32_t code) {
@@ -370,7 +369,7 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
 // publish each row's beta with its ready tag. The partials of a unit are contiguous
 // (1 KB per item) and come in by bulk copies of up to kMergeBatch items.
 __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, const MergeJob& u,
-                                           uint32_t& phase) {
+                                           float2 (*mbuf)[kMaxRows], uint32_t& phase) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   __threadfence();
@@ -388,7 +387,7 @@ __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, 
       fence_proxy_async();
       const uint32_t bytes = static_cast<uint32_t>(cnt) * kMaxRows * sizeof(float2);
       mbar_arrive_expect_tx(&ctl.merge_bar, bytes);
-      bulk_load(&ctl.mbuf[0][0], &P.partial[(u.item0 + s0) * kMaxRows], bytes, &ctl.merge_bar);
+      bulk_load(&mbuf[0][0], &P.partial[(u.item0 + s0) * kMaxRows], bytes, &ctl.merge_bar);
     }
     if (!warp_wait(&ctl.merge_bar, phase, P.wait_limit_ns, &ctl.abort)) return false;
     phase ^= 1u;
@@ -400,7 +399,7 @@ __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, 
       float2 e[kMergeBatch];
 #pragma unroll
       for (int j = 0; j < kMergeBatch; ++j) {
-        const float2 x = ctl.mbuf[j][row];
+        const float2 x = mbuf[j][row];
         e[j] = j < cnt ? x : make_float2(-INFINITY, 0.f);
       }
       float mb = M[k];
@@ -492,6 +491,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* qbuf = tiles;                             // kQBufs x 32 KB
   uint8_t* kbuf = tiles + kQBufs * kTileBytes;       // kKStages x 32 KB
+  // partials being merged (bulk-copy destination, 1 KB aligned)
+  float2 (*mbuf)[kMaxRows] = reinterpret_cast<float2 (*)[kMaxRows]>(kbuf + kKStages * kTileBytes);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -802,7 +803,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const MergeJob job = ctl.merge_job[ms];
       if (job.unit < 0) break;
-      if (!merge_unit(P, ctl, job, mphase)) {
+      if (!merge_unit(P, ctl, job, mbuf, mphase)) {
         set_error(P, ctl, 1u);
         // no bulk copy may still be writing shared memory when the CTA exits
         volatile int no_abort = 0;
