@@ -335,10 +335,42 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- sync warp
 
+// One round of loads of a unit's tagged normalisers (4 rows per lane); rows past n
+// read as ready.
+__device__ __forceinline__ void load_beta(const ScoreParams& P, int64_t unit, unsigned long long w[4]) {
+  const int r0 = 4 * (threadIdx.x & 31);
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    w[k] = (r0 + k < P.g.n_rows) ? __ldcg(&P.beta[unit * kMaxRows + r0 + k]) : (1ull << 32);
+}
+
+// If every row of w is tagged ready, stage -beta for the epilogue and return true.
+__device__ __forceinline__ bool stage_beta(const ScoreParams& P, ScoreCtl& ctl,
+                                           const unsigned long long w[4], uint32_t slot) {
+  const int lane = threadIdx.x & 31;
+  const int n = P.g.n_rows;
+  const int r0 = 4 * lane;
+  bool ready = true;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
+  if (!__all_sync(0xffffffffu, ready)) return false;
+  float4 b;
+  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
+  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
+  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
+  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
+  reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
+  return true;
+}
+
 // Phase-0 item: merge the two groups' (m, Z) per row, publish them and count the
-// item. Returns whether it was the unit's last item to arrive.
+// item. Returns whether it was the unit's last item to arrive. When the next ring
+// item is a phase-1 item not yet staged (next_unit >= 0), its normalisers are loaded
+// before the publication's fence and checked after its atomic (the round trips
+// overlap); *next_staged tells whether they were ready and are now staged.
 __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ctl,
-                                              const ItemDesc& d, uint32_t slot) {
+                                              const ItemDesc& d, uint32_t slot, int64_t next_unit,
+                                              uint32_t next_slot, bool* next_staged) {
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   float2 mz[4];
@@ -350,6 +382,8 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
   // the slot's shared data is in registers: hand the slot back to the producer
   __syncwarp();
   if (lane == 0) mbar_arrive(&ctl.item_empty[slot]);
+  unsigned long long w[4];
+  if (next_unit >= 0) load_beta(P, next_unit, w);
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     const int row = lane + 32 * k;
@@ -362,6 +396,7 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
     const uint32_t old = atomicAdd(&P.counts[d.unit], 1u);
     last = (old == static_cast<uint32_t>(d.splits - 1));
   }
+  *next_staged = next_unit >= 0 && stage_beta(P, ctl, w, next_slot);
   return __shfl_sync(0xffffffffu, last, 0) != 0;
 }
 
@@ -438,24 +473,9 @@ __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, 
 // the epilogue and true is returned.
 __device__ __forceinline__ bool try_stage_beta(const ScoreParams& P, ScoreCtl& ctl, int64_t unit,
                                                uint32_t slot) {
-  const int lane = threadIdx.x & 31;
-  const int n = P.g.n_rows;
-  const int r0 = 4 * lane;
   unsigned long long w[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k)
-    w[k] = (r0 + k < n) ? __ldcg(&P.beta[unit * kMaxRows + r0 + k]) : (1ull << 32);
-  bool ready = true;
-#pragma unroll
-  for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
-  if (!__all_sync(0xffffffffu, ready)) return false;
-  float4 b;
-  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
-  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
-  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
-  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
-  reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
-  return true;
+  load_beta(P, unit, w);
+  return stage_beta(P, ctl, w, slot);
 }
 
 // Phase-1 item: wait (bounded) for the unit's merged statistics and stage -beta.
@@ -738,6 +758,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t nslot = (it + 1) % kItemSlots;
         const uint32_t npar = ((it + 1) / kItemSlots) & 1u;
         bool next_checked = false;
+        int64_t next_unit = -1;   // the next item is a phase-1 item of this unit, not staged
         uint64_t t0 = 0;
         for (;;) {
           if (__all_sync(0xffffffffu, mbar_try_wait(&ctl.pub_full[slot], par))) break;
@@ -747,7 +768,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (pn < 0 || phn == 0) {
               next_checked = true;
             } else {
-              if (try_stage_beta(P, ctl, ctl.item_ring[nslot].unit, nslot)) {
+              next_unit = ctl.item_ring[nslot].unit;
+              if (try_stage_beta(P, ctl, next_unit, nslot)) {
+                next_unit = -1;
                 // the sync warp's whole part in that item is done: release it now
                 next_checked = next_staged = true;
                 __syncwarp();
@@ -769,7 +792,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
         }
-        if (ok && sync_rowstats(P, ctl, d, slot)) {           // hands the slot back early
+        bool late_staged = false;
+        const bool last = ok && sync_rowstats(P, ctl, d, slot, next_checked ? -1 : next_unit, nslot,
+                                              &late_staged);
+        if (late_staged) {
+          // staged after the publication: release that item now as well
+          next_staged = true;
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&ctl.beta_full[nslot]);
+            mbar_arrive(&ctl.item_empty[nslot]);
+          }
+        }
+        if (last) {                                              // the slot was handed back early
           MergeJob job;
           job.unit = d.unit;
           job.item0 = d.item0;
