@@ -389,7 +389,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     const uint32_t key = active ? ord_key(fmaf(lambda2, corr, my_st)) : 0u;
     const uint32_t wmax = __reduce_max_sync(0xffffffffu, key);
     const uint32_t wslot = __reduce_min_sync(0xffffffffu, (active && key == wmax) ? slot : 0xFFFFFFFFu);
-    const uint32_t wsec = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(slot) == wslot ? 0u : key);
+    // the runner-up only feeds the margins output
+    const uint32_t wsec =
+        margins ? __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(slot) == wslot ? 0u : key) : 0u;
     if (lane == 0) {
       sh.red[t & 1][warp][0] = wmax;
       sh.red[t & 1][warp][1] = wslot;
@@ -415,13 +417,13 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       if (margins) margins[t] = sec ? unord_key(best) - unord_key(sec) : INFINITY;
     }
     if (slot == js) active = false;
-    // dots of the warp's candidates with the admitted key (two accumulation chains
-    // per tile: even and odd k-steps)
-    float d[2][2][4];
+    // dots of the warp's candidates with the admitted key (four accumulation chains
+    // per tile: k-steps modulo 4)
+    float d[2][4][4];
 #pragma unroll
     for (int m = 0; m < 2; ++m)
 #pragma unroll
-      for (int c = 0; c < 2; ++c)
+      for (int c = 0; c < 4; ++c)
 #pragma unroll
         for (int e = 0; e < 4; ++e) d[m][c][e] = 0.f;
     uint32_t bf[8][2];
@@ -434,7 +436,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     for (int s8 = 0; s8 < 8; ++s8) {
 #pragma unroll
       for (int m = 0; m < 2; ++m) {
-        float* dd = d[m][s8 & 1];
+        float* dd = d[m][s8 & 3];
         asm volatile(
             "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
             "{%8,%9}, {%0,%1,%2,%3};"
@@ -444,8 +446,16 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       }
     }
     // rows g (element 0) and g + 8 (element 2) of tile t>>1; every column holds the same dot
-    const int mt = tq >> 1, el = (tq & 1) ? 2 : 0;
-    const float dot = d[mt][0][el] + d[mt][1][el];
+    // (register-only selection: no runtime index into d)
+    float dm[2][2];
+#pragma unroll
+    for (int m = 0; m < 2; ++m)
+#pragma unroll
+      for (int e = 0; e < 2; ++e)
+        dm[m][e] = (d[m][0][2 * e] + d[m][1][2 * e]) + (d[m][2][2 * e] + d[m][3][2 * e]);
+    const float dlo = (tq & 1) ? dm[0][1] : dm[0][0];
+    const float dhi = (tq & 1) ? dm[1][1] : dm[1][0];
+    const float dot = (tq >> 1) ? dhi : dlo;
     if (active) corr = fmaxf(corr, dot * my_inv * inv[js]);
   }
 
