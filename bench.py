@@ -39,8 +39,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "51b6660f9826d925d6e9327ed1c279162e393d3cca5c1ea293644a0b70007755",
-                 "bytes_per_launch": 2178510080 + 74864128}
+SCORE_TRAFFIC = {"source_sha256": "642e58bcb9f107cbf610fde5de9d3a4a83ff095db96c4fab55f505535f1966a6",
+                 "bytes_per_launch": 2171336192 + 74768896}
 
 
 def _score_source_sha():
