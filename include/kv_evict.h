@@ -33,13 +33,15 @@
  *      mu, sigma  packed per request: request r holds [N_L][Hkv][L_r] fp32 at
  *                 element offset N_L*Hkv*off_r
  *      indices    [n_req][N_L][Hkv][B] int32, kept candidate positions in
- *                 ascending order, -1 after the first min(B, Lc_r) entries
+ *                 ascending order, -1 after the first min(B_l, Lc_r) entries
+ *                 (B_l = B unless the plan has per-layer budgets, see
+ *                 kv_evict_plan_layered)
  *      order      [n_req][N_L][Hkv][B] int32, the same positions in admission
  *                 order (optional)
  *      margins    [n_req][N_L][Hkv][B] fp32, per admission the gap between the
  *                 best and the second-best greedy value (optional)
  *      k_out, v_out [n_req][N_L][Hkv][B+W][d] bf16: rows 0 .. m-1 are the kept
- *                 candidates in ascending position (m = min(B, Lc_r)), rows
+ *                 candidates in ascending position (m = min(B_l, Lc_r)), rows
  *                 m .. m+W-1 the W window tokens, remaining rows zero.
  *  * Every pointer must be 16-byte aligned; q_win and k additionally 128-byte.
  *  * stream is a cudaStream_t passed as void*. Every device call is
@@ -91,6 +93,16 @@ typedef struct kve_plan kve_plan;
 kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens,
                          int32_t n_req, kve_plan** plan_out,
                          size_t* workspace_bytes);
+
+/* kv_evict_plan with a budget per layer: layer_budgets is a HOST array [N_L] with
+ * 1 <= B_l <= cfg->budget; layer l keeps min(B_l, Lc_r) candidates (candidate pool
+ * min(factor * B_l, Lc_r)). cfg->budget stays the row stride of indices, order,
+ * margins (B) and of the compact cache (B + W). PyramidKV (Section 3.1) decreases
+ * the budget with depth while keeping the total of the uniform allocation; see
+ * kv_evict_budget_pyramid. layer_budgets = NULL is kv_evict_plan. */
+kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens,
+                                 int32_t n_req, const int32_t* layer_budgets,
+                                 kve_plan** plan_out, size_t* workspace_bytes);
 
 void kv_evict_plan_destroy(kve_plan* plan);
 
@@ -161,6 +173,17 @@ kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream);
  * Writes lambda_out[num_layers]. */
 kve_status kv_evict_profile(int32_t kind, const float* c, int32_t num_layers,
                             const int32_t* seg_bounds, float* lambda_out);
+
+/* A depth-decreasing budget schedule with the total of the uniform one (Section 3.1
+ * states only these two properties of PyramidKV's allocation; this function is a
+ * reading of it): budgets_out[l] (HOST, [num_layers]) falls linearly with depth
+ * from 2B - b to b, b = max(1, floor(last_ratio * B)), rounded down and the
+ * remainder given one each to the shallowest layers, so that the budgets are
+ * non-increasing and sum to num_layers * B. last_ratio = 1 is uniform. The
+ * largest budget is budgets_out[0]: pass it as cfg->budget. Returns KVE_EINVAL
+ * unless B >= 1, num_layers >= 1 and 0 < last_ratio <= 1. */
+kve_status kv_evict_budget_pyramid(int32_t budget, int32_t num_layers,
+                                   float last_ratio, int32_t* budgets_out);
 
 const char* kv_evict_strerror(kve_status status);
 

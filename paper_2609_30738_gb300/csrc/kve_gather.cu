@@ -2,8 +2,8 @@
 // keeps B cached entries; the W window tokens are kept as well).
 //
 // Unit u's compact cache is [B + W][d]: rows 0 .. m-1 are the kept candidates in
-// ascending position (m = min(B, Lc)), rows m .. m+W-1 the window tokens
-// Lc .. L-1, the rest zero. A row is 256 bytes, copied by 16 lanes with 16-byte
+// ascending position (m = min(B_l, Lc), B_l the unit's layer budget), rows
+// m .. m+W-1 the window tokens Lc .. L-1, the rest zero. A row is 256 bytes, copied by 16 lanes with 16-byte
 // accesses, key and value alike; the copy is bit-exact.
 #include "kve_internal.h"
 
@@ -17,7 +17,7 @@ __global__ void __launch_bounds__(kGatherThreads) gather_kernel(const __grid_con
   const int W = P.g.window;
   const int B = P.budget;
   const int Lc = u.L - W;
-  const int m = min(B, Lc);
+  const int m = min(P.layer_budget[u.layer], Lc);
   const int rows = B + W;
   const int half = threadIdx.x >> 4;            // 16 rows in flight per block
   const int lane16 = threadIdx.x & 15;

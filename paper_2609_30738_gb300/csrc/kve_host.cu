@@ -100,6 +100,12 @@ extern "C" {
 
 kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t n_req,
                          kve_plan** plan_out, size_t* workspace_bytes) {
+  return kv_evict_plan_layered(cfg, seq_lens, n_req, nullptr, plan_out, workspace_bytes);
+}
+
+kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens, int32_t n_req,
+                                 const int32_t* layer_budgets, kve_plan** plan_out,
+                                 size_t* workspace_bytes) {
   if (!cfg || !seq_lens || !plan_out) return KVE_EINVAL;
   *plan_out = nullptr;
   const kve_config& c = *cfg;
@@ -117,6 +123,14 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
   if (!plan) return KVE_ENOMEM;
   std::memset(plan, 0, sizeof(*plan));
   plan->cfg = c;
+  for (int l = 0; l < c.num_layers; ++l) {
+    const int32_t b = layer_budgets ? layer_budgets[l] : c.budget;
+    if (b < 1 || b > c.budget) {
+      delete plan;
+      return KVE_EINVAL;
+    }
+    plan->layer_budget[l] = b;
+  }
   plan->wait_limit_ns = kDefaultWaitNs;
   plan->fault = 0;
   kve::Geometry& g = plan->geo;
@@ -238,6 +252,7 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
     if (!std::isfinite(lambda1[l]) || !std::isfinite(lambda2[l])) return KVE_EINVAL;
     p.lambda1[l] = lambda1[l];
     p.lambda2[l] = lambda2[l];
+    p.layer_budget[l] = plan->layer_budget[l];
   }
   p.mu = mu;
   p.sigma = sigma;
@@ -257,6 +272,7 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16
   std::memset(&p, 0, sizeof(p));
   p.g = plan->geo;
   p.budget = plan->cfg.budget;
+  for (int l = 0; l < plan->geo.num_layers; ++l) p.layer_budget[l] = plan->layer_budget[l];
   p.k = k;
   p.v = v;
   p.indices = indices;
@@ -299,6 +315,30 @@ kve_status kv_evict_profile(int32_t kind, const float* c, int32_t num_layers, co
     }
     lambda_out[l] = static_cast<float>(std::sinh(a));
   }
+  return KVE_OK;
+}
+
+kve_status kv_evict_budget_pyramid(int32_t budget, int32_t num_layers, float last_ratio,
+                                   int32_t* budgets_out) {
+  if (!budgets_out || budget < 1 || num_layers < 1 || !(last_ratio > 0.f) || last_ratio > 1.f)
+    return KVE_EINVAL;
+  const int64_t N = num_layers, total = N * budget;
+  if (N == 1) {
+    budgets_out[0] = budget;
+    return KVE_OK;
+  }
+  // linear in depth from top to bottom = max(1, floor(r*B)), top = 2B - bottom, so the
+  // mean is B; the floors' shortfall goes to the shallowest layers, one each
+  const int64_t bottom = std::max<int64_t>(1, static_cast<int64_t>(std::floor(last_ratio * budget)));
+  const int64_t top = 2 * static_cast<int64_t>(budget) - bottom;
+  int64_t sum = 0;
+  for (int64_t l = 0; l < N; ++l) {
+    // floor of the linear interpolation: never above it, so sum <= total
+    const int64_t b = bottom + ((top - bottom) * (N - 1 - l)) / (N - 1);
+    budgets_out[l] = static_cast<int32_t>(b);
+    sum += b;
+  }
+  for (int64_t l = 0; sum < total; l = (l + 1) % N, ++sum) ++budgets_out[l];
   return KVE_OK;
 }
 

@@ -113,7 +113,8 @@ struct ScoreParams {
 
 struct SelectParams {
   Geometry g;
-  int32_t budget, pool_kernel, cand_factor;
+  int32_t budget;            // row stride of indices / order / margins (the plan's B)
+  int32_t pool_kernel, cand_factor;
   float norm_eps;
   const float* mu;
   const float* sigma;
@@ -124,11 +125,13 @@ struct SelectParams {
   uint32_t* keys;            // workspace scratch
   float lambda1[kMaxLayers];
   float lambda2[kMaxLayers];
+  int32_t layer_budget[kMaxLayers];   // B_l <= budget kept candidates of layer l
 };
 
 struct GatherParams {
   Geometry g;
-  int32_t budget;
+  int32_t budget;            // row stride: B + W rows per unit
+  int32_t layer_budget[kMaxLayers];
   const uint16_t* k;
   const uint16_t* v;
   const int32_t* indices;
@@ -140,6 +143,7 @@ struct GatherParams {
 
 struct kve_plan {
   kve_config cfg;
+  int32_t layer_budget[kve::kMaxLayers];   // B_l per layer (all cfg.budget by default)
   kve::Geometry geo;
   kve::WsLayout ws;
   uint64_t wait_limit_ns;

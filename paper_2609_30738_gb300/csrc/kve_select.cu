@@ -100,9 +100,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   const UnitInfo u = unit_info(P.g, blockIdx.x);
   const int W = P.g.window;
   const int Lc = u.L - W;
-  const int B = P.budget;
-  const int C = P.cand_factor == 0 ? Lc : min(P.cand_factor * B, Lc);
-  const int nsel = min(B, C);
+  const int B = P.budget;                     // row stride of the outputs
+  const int Bl = P.layer_budget[u.layer];     // this layer's budget, <= B
+  const int C = P.cand_factor == 0 ? Lc : min(P.cand_factor * Bl, Lc);
+  const int nsel = min(Bl, C);
   const float lambda1 = P.lambda1[u.layer];
   const float lambda2 = P.lambda2[u.layer];
   const float* mu = P.mu + u.mu_off;
@@ -574,6 +575,7 @@ extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float*
     if (!isfinite(lambda1[l]) || !isfinite(lambda2[l])) return KVE_EINVAL;
     p.lambda1[l] = lambda1[l];
     p.lambda2[l] = lambda2[l];
+    p.layer_budget[l] = plan->layer_budget[l];
   }
   p.mu = mu;
   p.sigma = sigma;

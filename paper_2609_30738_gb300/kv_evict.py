@@ -18,9 +18,9 @@ LIB_PATH = os.path.join(_HERE, "libkvevict.so")
 KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 
 # Names declared in include/kv_evict.h.
-EXPORTS = ("kv_evict_plan", "kv_evict_plan_destroy", "kv_evict_plan_set_debug", "kv_evict_score",
-           "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather", "kv_evict_status",
-           "kv_evict_profile", "kv_evict_strerror")
+EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_destroy", "kv_evict_plan_set_debug",
+           "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather",
+           "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
 
 
 class KvEvictError(RuntimeError):
@@ -50,6 +50,9 @@ def _lib():
         vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
         lib.kv_evict_plan.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32,
                                       ctypes.POINTER(vp), ctypes.POINTER(ctypes.c_size_t)]
+        lib.kv_evict_plan_layered.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32, vp,
+                                              ctypes.POINTER(vp), ctypes.POINTER(ctypes.c_size_t)]
+        lib.kv_evict_budget_pyramid.argtypes = [i32, i32, ctypes.c_float, vp]
         lib.kv_evict_plan_destroy.argtypes = [vp]
         lib.kv_evict_plan_destroy.restype = None
         lib.kv_evict_plan_set_debug.argtypes = [vp, ctypes.c_uint64, i32]
@@ -61,9 +64,9 @@ def _lib():
         lib.kv_evict_profile.argtypes = [i32, vp, i32, vp, vp]
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
         lib.kv_evict_strerror.restype = ctypes.c_char_p
-        for name in ("kv_evict_plan", "kv_evict_plan_set_debug", "kv_evict_score", "kv_evict_select",
-                     "kv_evict_select_noalloc", "kv_evict_gather", "kv_evict_status",
-                     "kv_evict_profile"):
+        for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_set_debug",
+                     "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather",
+                     "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
             getattr(lib, name).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -103,9 +106,10 @@ def make_config(spec: dict) -> Config:
 
 
 class Plan:
-    """kv_evict_plan for a configuration and the prefix lengths of the requests."""
+    """kv_evict_plan (kv_evict_plan_layered when layer_budgets is given) for a
+    configuration and the prefix lengths of the requests."""
 
-    def __init__(self, spec: dict, seq_lens):
+    def __init__(self, spec: dict, seq_lens, layer_budgets=None):
         lib = _lib()
         self.spec = dict(spec)
         self.seq_lens = [int(x) for x in seq_lens]
@@ -113,8 +117,16 @@ class Plan:
         lens = (ctypes.c_int64 * len(self.seq_lens))(*self.seq_lens)
         handle = ctypes.c_void_p()
         ws = ctypes.c_size_t()
-        _check(lib.kv_evict_plan(ctypes.byref(self._cfg), lens, len(self.seq_lens),
-                                 ctypes.byref(handle), ctypes.byref(ws)), "kv_evict_plan")
+        if layer_budgets is None:
+            self.layer_budgets = [int(spec["budget"])] * int(spec["num_layers"])
+            _check(lib.kv_evict_plan(ctypes.byref(self._cfg), lens, len(self.seq_lens),
+                                     ctypes.byref(handle), ctypes.byref(ws)), "kv_evict_plan")
+        else:
+            self.layer_budgets = [int(b) for b in layer_budgets]
+            lb = np.ascontiguousarray(self.layer_budgets, dtype=np.int32)
+            _check(lib.kv_evict_plan_layered(ctypes.byref(self._cfg), lens, len(self.seq_lens),
+                                             lb.ctypes.data, ctypes.byref(handle), ctypes.byref(ws)),
+                   "kv_evict_plan_layered")
         self._h = handle
         self.workspace_bytes = ws.value
 
@@ -183,6 +195,14 @@ def profile(kind: str, c, num_layers: int, seg_bounds=None) -> np.ndarray:
     _check(_lib().kv_evict_profile(k, cc.ctypes.data, num_layers,
                                    None if sb is None else sb.ctypes.data, out.ctypes.data),
            "kv_evict_profile")
+    return out
+
+
+def budget_pyramid(budget: int, num_layers: int, last_ratio: float) -> np.ndarray:
+    """kv_evict_budget_pyramid: a depth-decreasing schedule with the uniform total."""
+    out = np.zeros(num_layers, dtype=np.int32)
+    _check(_lib().kv_evict_budget_pyramid(int(budget), int(num_layers), float(last_ratio),
+                                          out.ctypes.data), "kv_evict_budget_pyramid")
     return out
 
 

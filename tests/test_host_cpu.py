@@ -83,3 +83,39 @@ def test_profile_matches_oracle(kind, c, N):
     lib_vals = K.profile(kind, c, N)
     ref = O.depth_profile(kind, c, N)
     np.testing.assert_allclose(lib_vals, ref, rtol=2e-7, atol=1e-7)
+
+
+@pytest.mark.parametrize("B,N,r", [(64, 32, 0.5), (64, 32, 1.0), (64, 32, 0.1), (32, 5, 0.3),
+                                   (1, 4, 1.0), (7, 3, 0.2), (128, 1, 0.5), (16, 2, 0.25)])
+def test_budget_pyramid_properties(B, N, r):
+    """Depth-decreasing budgets with the uniform total: non-increasing, sum N*B,
+    first >= B >= last >= 1, last near r*B, uniform for r = 1."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    b = K.budget_pyramid(B, N, r).astype(np.int64)
+    assert b.sum() == N * B
+    assert np.all(np.diff(b) <= 0) and b.min() >= 1
+    assert b[0] >= B >= b[-1]
+    if N > 1:
+        assert abs(b[-1] - max(1, int(np.floor(r * B)))) <= 1
+        # linear in depth: second differences of at most one unit (rounding)
+        assert np.all(np.abs(np.diff(b, 2)) <= 2)
+    if r == 1.0:
+        assert np.all(b == B)
+
+
+def test_budget_pyramid_and_layered_plan_validation():
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    for args in [(0, 4, 0.5), (64, 0, 0.5), (64, 4, 0.0), (64, 4, 1.5)]:
+        with pytest.raises(K.KvEvictError) as e:
+            K.budget_pyramid(*args)
+        assert e.value.status == K.KVE_EINVAL
+    spec = _spec(num_layers=4, budget=24)
+    p = K.Plan(spec, [2048], layer_budgets=[24, 18, 14, 8])
+    assert p.layer_budgets == [24, 18, 14, 8]
+    assert p.workspace_bytes == K.Plan(spec, [2048]).workspace_bytes
+    for lb in ([24, 25, 14, 8], [24, 18, 0, 8]):          # above the stride, below one
+        with pytest.raises(K.KvEvictError) as e:
+            K.Plan(spec, [2048], layer_budgets=lb)
+        assert e.value.status == K.KVE_EINVAL

@@ -25,9 +25,9 @@ def _lib():
     return K
 
 
-def _run(spec, batch, lambdas=None):
+def _run(spec, batch, lambdas=None, layer_budgets=None):
     from paper_2609_30738_gb300 import kv_evict as K
-    plan = K.Plan(spec, batch["seq_lens"])
+    plan = K.Plan(spec, batch["seq_lens"], layer_budgets=layer_budgets)
     bufs = K.Buffers(plan)
     if lambdas is None:
         lambdas = lambda_arrays(spec, K.profile)
@@ -69,7 +69,8 @@ def _check_units(spec, batch, plan, bufs, lambdas, units, sel_mode="replay"):
         tag = f"unit(r={r},l={layer},h={h})"
         worst = max(worst, PT.check_mu_sigma(mu_all[o:o + L], sg_all[o:o + L], mu_ref, sg_ref, tag))
         ui = _unit_index(spec, seq, r, layer, h)
-        swaps += PT.check_selection(ord_all[ui], idx_all[ui], mu_ref, sg_ref, kf, L, W, B,
+        Bl = plan.layer_budgets[layer]
+        swaps += PT.check_selection(ord_all[ui], idx_all[ui], mu_ref, sg_ref, kf, L, W, Bl,
                                     float(lambdas[0][layer]), float(lambdas[1][layer]),
                                     spec["pool_kernel"], spec["candidate_factor"],
                                     spec["norm_eps"], margins_gpu=mar_all[ui], what=tag)
@@ -109,6 +110,25 @@ def test_window8_partial_rows():
     batch = synth.make_batch(spec, seed=8)
     plan, bufs, _, lam = _run(spec, batch)
     _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
+def test_layer_budgets_pyramid_every_unit():
+    """Per-layer budgets (a depth-decreasing schedule with the uniform total): every
+    unit's selection against the oracle at its layer's budget, the compact cache at
+    the plan's row stride."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=4, budget=40,
+                  seq_lens=[1500, 300, 2100])
+    lb = K.budget_pyramid(24, 4, 0.4)            # mean 24, deepest layer ~ 9
+    assert lb[0] <= spec["budget"] and lb.sum() == 4 * 24
+    batch = synth.make_batch(spec, seed=13)
+    plan, bufs, _, lam = _run(spec, batch, layer_budgets=lb)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+    # uniform budgets through the layered entry point equal the plain plan bit for bit
+    plan_u, bufs_u, _, _ = _run(spec, batch, lambdas=lam, layer_budgets=[spec["budget"]] * 4)
+    plan_p, bufs_p, _, _ = _run(spec, batch, lambdas=lam)
+    assert torch.equal(bufs_u.indices, bufs_p.indices)
+    assert torch.equal(bufs_u.k_out, bufs_p.k_out)
 
 
 @pytest.mark.parametrize("lams", [(0.0, 0.0), (0.0, -0.15), (0.5, 0.6), (-0.3, -0.5), (2.0, -3.6)])
