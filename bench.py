@@ -39,8 +39,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "642e58bcb9f107cbf610fde5de9d3a4a83ff095db96c4fab55f505535f1966a6",
-                 "bytes_per_launch": 2171336192 + 74768896}
+SCORE_TRAFFIC = {"source_sha256": "124d6003395a65bd4e61eec57fcf041e3a6206c79d51b6b7ff4863ee99248673",
+                 "bytes_per_launch": 2178174720 + 74808576}
 
 
 def _score_source_sha():
