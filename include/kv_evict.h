@@ -134,6 +134,29 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu,
                            int32_t* indices, int32_t* order, float* margins,
                            void* ws, void* stream);
 
+/* Step 3 for n_profiles profiles of the layer-wise coefficients in one pass over
+ * the units (Section 3.3 searches over profiles and re-selects for each; mu and
+ * sigma do not depend on the coefficients, so one kv_evict_score serves them all).
+ * lambda1 and lambda2 are HOST arrays [n_profiles][N_L]; profile p selects exactly
+ * what kv_evict_select selects with lambda1 + p*N_L and lambda2 + p*N_L. Outputs are
+ * stacked by profile: indices [n_profiles][n_units][B]; order and margins likewise
+ * (either may be NULL). ws is a separate scratch buffer (256-byte aligned) of
+ * kv_evict_select_profiles_workspace bytes, not the plan's workspace. One launch
+ * carries 6144 / (2 N_L) profiles (96 for N_L = 32); more go to further launches on
+ * stream. Returns KVE_EINVAL for n_profiles < 1 or a non-finite coefficient, before
+ * any launch. */
+kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles,
+                                    const float* mu, const float* sigma,
+                                    const uint16_t* k, const float* lambda1,
+                                    const float* lambda2, int32_t* indices,
+                                    int32_t* order, float* margins, void* ws,
+                                    void* stream);
+
+/* *bytes = scratch of kv_evict_select_profiles for n_profiles profiles (4 bytes per
+ * prefix token per unit per profile). */
+kve_status kv_evict_select_profiles_workspace(const kve_plan* plan,
+                                              int32_t n_profiles, size_t* bytes);
+
 /* Step 3 without a workspace. The paper has no counterpart: this entry point
  * exists for callers that cannot allocate device memory at eviction time --
  * serving engines that reserve nearly all of HBM for their own KV-cache pool and

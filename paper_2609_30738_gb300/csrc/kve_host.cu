@@ -235,33 +235,105 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
                                                                                         : KVE_ECUDA;
 }
 
+}  // extern "C"
+
+namespace {
+
+// The select kernel's parameters common to every entry point; lambda1 / lambda2
+// (HOST [N_L]) may be NULL when a profile table supplies the coefficients.
+kve_status select_params(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
+                         const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
+                         float* margins, kve::SelectParams* p) {
+  const kve::Geometry& g = plan->geo;
+  std::memset(p, 0, sizeof(*p));
+  p->g = g;
+  p->budget = plan->cfg.budget;
+  p->pool_kernel = plan->cfg.pool_kernel;
+  p->cand_factor = plan->cfg.candidate_factor;
+  p->norm_eps = plan->cfg.norm_eps;
+  for (int l = 0; l < g.num_layers; ++l) {
+    if (lambda1 && (!std::isfinite(lambda1[l]) || !std::isfinite(lambda2[l]))) return KVE_EINVAL;
+    p->lambda1[l] = lambda1 ? lambda1[l] : 0.f;
+    p->lambda2[l] = lambda2 ? lambda2[l] : 0.f;
+    p->layer_budget[l] = plan->layer_budget[l];
+  }
+  p->mu = mu;
+  p->sigma = sigma;
+  p->k = k;
+  p->indices = indices;
+  p->order = order;
+  p->margins = margins;
+  return KVE_OK;
+}
+
+// Scratch words of one profile (the ordered base score of every prefix token of
+// every unit), padded to 256 bytes.
+int64_t profile_keys_words(const kve_plan* plan) {
+  const kve::Geometry& g = plan->geo;
+  const int64_t words = static_cast<int64_t>(g.num_layers) * g.hkv * g.total_tokens;
+  return (words + 63) / 64 * 64;
+}
+
+// Profiles one launch can carry in its parameter table.
+int32_t profiles_per_launch(const kve_plan* plan) {
+  return kve::kProfileLambdas / (2 * plan->geo.num_layers);
+}
+
+}  // namespace
+
+extern "C" {
+
 kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
                            const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
                            float* margins, void* ws, void* stream) {
   if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws) return KVE_EINVAL;
   if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
-  const kve::Geometry& g = plan->geo;
   kve::SelectParams p;
-  std::memset(&p, 0, sizeof(p));
-  p.g = g;
-  p.budget = plan->cfg.budget;
-  p.pool_kernel = plan->cfg.pool_kernel;
-  p.cand_factor = plan->cfg.candidate_factor;
-  p.norm_eps = plan->cfg.norm_eps;
-  for (int l = 0; l < g.num_layers; ++l) {
-    if (!std::isfinite(lambda1[l]) || !std::isfinite(lambda2[l])) return KVE_EINVAL;
-    p.lambda1[l] = lambda1[l];
-    p.lambda2[l] = lambda2[l];
-    p.layer_budget[l] = plan->layer_budget[l];
-  }
-  p.mu = mu;
-  p.sigma = sigma;
-  p.k = k;
-  p.indices = indices;
-  p.order = order;
-  p.margins = margins;
+  const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
+  if (s != KVE_OK) return s;
   p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.keys);
   return kve::launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}
+
+kve_status kv_evict_select_profiles_workspace(const kve_plan* plan, int32_t n_profiles, size_t* bytes) {
+  if (!plan || !bytes || n_profiles < 1) return KVE_EINVAL;
+  *bytes = static_cast<size_t>(n_profiles) * static_cast<size_t>(profile_keys_words(plan)) * sizeof(uint32_t);
+  return KVE_OK;
+}
+
+kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles, const float* mu,
+                                    const float* sigma, const uint16_t* k, const float* lambda1,
+                                    const float* lambda2, int32_t* indices, int32_t* order, float* margins,
+                                    void* ws, void* stream) {
+  if (!plan || n_profiles < 1 || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws)
+    return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
+  const int32_t nl = plan->geo.num_layers;
+  for (int64_t i = 0; i < static_cast<int64_t>(n_profiles) * nl; ++i)
+    if (!std::isfinite(lambda1[i]) || !std::isfinite(lambda2[i])) return KVE_EINVAL;
+  kve::SelectParams p;
+  const kve_status s = select_params(plan, mu, sigma, k, nullptr, nullptr, indices, order, margins, &p);
+  if (s != KVE_OK) return s;
+  p.keys = static_cast<uint32_t*>(ws);
+  // the table rides in the kernel parameters; profiles beyond its capacity go to
+  // further launches on the same stream
+  static thread_local kve::ProfileTable table;
+  table.pad = 0;
+  table.keys_stride = profile_keys_words(plan);
+  table.out_stride = plan->geo.n_units * static_cast<int64_t>(plan->cfg.budget);
+  const int32_t cap = profiles_per_launch(plan);
+  for (int32_t f = 0; f < n_profiles; f += cap) {
+    const int32_t cnt = std::min(cap, n_profiles - f);
+    table.first = f;
+    for (int32_t j = 0; j < cnt; ++j)
+      for (int32_t l = 0; l < nl; ++l) {
+        table.lam[(2 * j) * nl + l] = lambda1[static_cast<int64_t>(f + j) * nl + l];
+        table.lam[(2 * j + 1) * nl + l] = lambda2[static_cast<int64_t>(f + j) * nl + l];
+      }
+    if (kve::launch_select_profiles(*plan, p, table, cnt, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+      return KVE_ECUDA;
+  }
+  return KVE_OK;
 }
 
 kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16_t* v, const int32_t* indices,

@@ -128,6 +128,20 @@ struct SelectParams {
   int32_t layer_budget[kMaxLayers];   // B_l <= budget kept candidates of layer l
 };
 
+// Coefficient profiles of one multi-profile selection launch (kernel parameter):
+// profile first + y of the launch (grid y) uses lam[2*y*N_L + l] (lambda1) and
+// lam[(2*y + 1)*N_L + l] (lambda2) on layer l, scratch keys + (first + y) *
+// keys_stride and outputs + (first + y) * out_stride.
+constexpr int kProfileLambdas = 6144;   // 24 KB of coefficients per launch
+struct ProfileTable {
+  static constexpr bool kMulti = true;
+  int32_t first;
+  int32_t pad;
+  int64_t keys_stride;       // scratch words per profile
+  int64_t out_stride;        // output elements per profile (n_units * B)
+  float lam[kProfileLambdas];
+};
+
 struct GatherParams {
   Geometry g;
   int32_t budget;            // row stride: B + W rows per unit
@@ -155,5 +169,7 @@ namespace kve {
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                          const ScoreParams& p, int ctas, cudaStream_t stream);
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
+cudaError_t launch_select_profiles(const kve_plan& plan, const SelectParams& p, const ProfileTable& table,
+                                   int profiles, cudaStream_t stream);
 cudaError_t launch_gather(const kve_plan& plan, const GatherParams& p, cudaStream_t stream);
 }  // namespace kve

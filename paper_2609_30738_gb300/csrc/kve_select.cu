@@ -16,7 +16,10 @@
 //     both corr(i, {}) and the clamp at 0);
 //  5. write the admitted positions ascending (and optionally in admission order,
 //     with the best-minus-second margin of every admission).
-// The block has one thread per pool slot (256 for C <= 256, else 512).
+// The block has one thread per pool slot (256 for C <= 256, else 512). A launch for
+// several coefficient profiles (Section 3.3 re-selects for every profile a search
+// tries; mu and sigma do not depend on them) runs one CTA per (unit, profile), the
+// profile's coefficients and scratch taken from a table in the kernel parameters.
 #include <mutex>
 
 #include "kve_internal.h"
@@ -90,8 +93,15 @@ __device__ __forceinline__ uint32_t block_excl_suffix(uint32_t x, SelSmall<NT>& 
   return incl - x + after;
 }
 
-template <int NT>
-__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams P) {
+// The coefficients of one selection: those of SelectParams (kMulti = false), or
+// profile first + blockIdx.y of a table (kMulti = true).
+struct OneProfile {
+  static constexpr bool kMulti = false;
+};
+
+template <int NT, class Prof>
+__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams P,
+                                                    const __grid_constant__ Prof prof) {
   __shared__ SelSmall<NT> sh;
   extern __shared__ __align__(16) uint8_t dyn[];
   const int tid = threadIdx.x;
@@ -104,11 +114,19 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   const int Bl = P.layer_budget[u.layer];     // this layer's budget, <= B
   const int C = P.cand_factor == 0 ? Lc : min(P.cand_factor * Bl, Lc);
   const int nsel = min(Bl, C);
-  const float lambda1 = P.lambda1[u.layer];
-  const float lambda2 = P.lambda2[u.layer];
+  float lambda1 = P.lambda1[u.layer];
+  float lambda2 = P.lambda2[u.layer];
+  int64_t keys_off = 0, out_off = 0;   // this profile's scratch and output blocks
+  if constexpr (Prof::kMulti) {
+    const int row = 2 * static_cast<int>(blockIdx.y) * P.g.num_layers + u.layer;
+    lambda1 = prof.lam[row];
+    lambda2 = prof.lam[row + P.g.num_layers];
+    keys_off = static_cast<int64_t>(prof.first + blockIdx.y) * prof.keys_stride;
+    out_off = static_cast<int64_t>(prof.first + blockIdx.y) * prof.out_stride;
+  }
   const float* mu = P.mu + u.mu_off;
   const float* sg = P.sigma + u.mu_off;
-  uint32_t* keys = P.keys + u.mu_off;
+  uint32_t* keys = P.keys + keys_off + u.mu_off;
   const int h = P.pool_kernel / 2;
 
   // shared memory: [ big | spos | cpos | st | inv ]; `big` holds in turn the pooling
@@ -384,8 +402,8 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       afr[m][s8][3] = r1 < C ? kw[r1 * 64 + 8 * s8 + tq + 4] : 0u;
     }
   }
-  int32_t* order = P.order ? P.order + u.unit * B : nullptr;
-  float* margins = P.margins ? P.margins + u.unit * B : nullptr;
+  int32_t* order = P.order ? P.order + out_off + u.unit * B : nullptr;
+  float* margins = P.margins ? P.margins + out_off + u.unit * B : nullptr;
   for (int t = 0; t < nsel; ++t) {
     const uint32_t key = active ? ord_key(fmaf(lambda2, corr, my_st)) : 0u;
     const uint32_t wmax = __reduce_max_sync(0xffffffffu, key);
@@ -468,7 +486,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   const bool sel = tid < C && cpos[tid] != 0;
   uint32_t tot;
   const uint32_t rank = block_excl_count<NT>(sel, sh, &tot);
-  int32_t* out = P.indices + u.unit * B;
+  int32_t* out = P.indices + out_off + u.unit * B;
   if (sel) out[rank] = spos[tid];
   for (int r = nsel + tid; r < B; r += NT) out[r] = -1;
   if (order)
@@ -486,29 +504,43 @@ static_assert(kChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histog
 static_assert(kChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
               "pool tiles fit");
 static_assert(kChunks * 256 * sizeof(uint4) >= kTieCap * sizeof(int32_t), "tie list fits");
+// both parameter blocks of a multi-profile launch fit the 32764-byte kernel
+// parameter space
+static_assert(sizeof(SelectParams) + sizeof(ProfileTable) + 64 <= 32764, "profile table fits");
 
 }  // namespace
 
-cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {
+template <class Prof>
+cudaError_t launch_select_grid(const kve_plan& plan, const SelectParams& p, const Prof& prof,
+                               unsigned profiles, cudaStream_t stream) {
   // pool size bound: the largest C over the requests
   int max_lc = 0;
   for (int r = 0; r < plan.geo.n_req; ++r) max_lc = max(max_lc, plan.geo.req_len[r] - plan.geo.window);
   const int cmax = p.cand_factor == 0 ? max_lc : min(p.cand_factor * p.budget, max_lc);
-  const unsigned grid = static_cast<unsigned>(plan.geo.n_units);
+  const dim3 grid(static_cast<unsigned>(plan.geo.n_units), profiles);
   if (cmax <= 256) {
     constexpr size_t smem = select_smem<256>();
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<256, Prof>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    select_kernel<256><<<grid, 256, smem, stream>>>(p);
+    select_kernel<256, Prof><<<grid, 256, smem, stream>>>(p, prof);
   } else {
     constexpr size_t smem = select_smem<512>();
-    cudaError_t e = cudaFuncSetAttribute(select_kernel<512>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+    cudaError_t e = cudaFuncSetAttribute(select_kernel<512, Prof>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    select_kernel<512><<<grid, 512, smem, stream>>>(p);
+    select_kernel<512, Prof><<<grid, 512, smem, stream>>>(p, prof);
   }
   return cudaGetLastError();
+}
+
+cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {
+  return launch_select_grid(plan, p, OneProfile{}, 1u, stream);
+}
+
+cudaError_t launch_select_profiles(const kve_plan& plan, const SelectParams& p, const ProfileTable& table,
+                                   int profiles, cudaStream_t stream) {
+  return launch_select_grid(plan, p, table, static_cast<unsigned>(profiles), stream);
 }
 
 }  // namespace kve

@@ -19,7 +19,8 @@ KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 
 # Names declared in include/kv_evict.h.
 EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_destroy", "kv_evict_plan_set_debug",
-           "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather",
+           "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
+           "kv_evict_select_profiles_workspace", "kv_evict_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
 
 
@@ -59,13 +60,16 @@ def _lib():
         lib.kv_evict_score.argtypes = [vp] * 7
         lib.kv_evict_select.argtypes = [vp] * 11
         lib.kv_evict_select_noalloc.argtypes = [vp] * 10
+        lib.kv_evict_select_profiles.argtypes = [vp, i32] + [vp] * 10
+        lib.kv_evict_select_profiles_workspace.argtypes = [vp, i32, vp]
         lib.kv_evict_gather.argtypes = [vp] * 7
         lib.kv_evict_status.argtypes = [vp, vp, vp]
         lib.kv_evict_profile.argtypes = [i32, vp, i32, vp, vp]
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
         lib.kv_evict_strerror.restype = ctypes.c_char_p
         for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_set_debug",
-                     "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_gather",
+                     "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc",
+                     "kv_evict_select_profiles", "kv_evict_select_profiles_workspace", "kv_evict_gather",
                      "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
             getattr(lib, name).restype = ctypes.c_int
         _LIB = lib
@@ -175,6 +179,27 @@ class Plan:
                                               l1.ctypes.data, l2.ctypes.data, _ptr(indices),
                                               _ptr(order), _ptr(margins), _stream_ptr(stream)),
                "kv_evict_select_noalloc")
+
+    def select_profiles_workspace(self, n_profiles: int) -> int:
+        """Bytes of scratch that select_profiles needs for n_profiles profiles."""
+        out = ctypes.c_size_t(0)
+        _check(_lib().kv_evict_select_profiles_workspace(self._h, int(n_profiles), ctypes.byref(out)),
+               "kv_evict_select_profiles_workspace")
+        return out.value
+
+    def select_profiles(self, mu, sigma, k, lambda1, lambda2, indices, ws, order=None, margins=None,
+                        stream=None):
+        """Selection for P coefficient profiles at once: lambda1 / lambda2 are
+        [P, N_L]; indices (and order / margins) are [P, n_units, B]; ws holds
+        select_profiles_workspace(P) bytes."""
+        l1 = np.ascontiguousarray(lambda1, dtype=np.float32)
+        l2 = np.ascontiguousarray(lambda2, dtype=np.float32)
+        assert l1.ndim == 2 and l1.shape[1] == self.spec["num_layers"] and l2.shape == l1.shape
+        _check(_lib().kv_evict_select_profiles(self._h, int(l1.shape[0]), _ptr(mu), _ptr(sigma), _ptr(k),
+                                               l1.ctypes.data, l2.ctypes.data, _ptr(indices),
+                                               _ptr(order), _ptr(margins), _ptr(ws),
+                                               _stream_ptr(stream)),
+               "kv_evict_select_profiles")
 
     def gather(self, k, v, indices, k_out, v_out, stream=None):
         _check(_lib().kv_evict_gather(self._h, _ptr(k), _ptr(v), _ptr(indices), _ptr(k_out),

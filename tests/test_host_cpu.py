@@ -119,3 +119,29 @@ def test_budget_pyramid_and_layered_plan_validation():
         with pytest.raises(K.KvEvictError) as e:
             K.Plan(spec, [2048], layer_budgets=lb)
         assert e.value.status == K.KVE_EINVAL
+
+
+def test_select_profiles_validation_without_gpu():
+    """Multi-profile selection: scratch size per profile, and the host checks that
+    return before any launch (so fake, aligned device addresses suffice)."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    lib = K.library()
+    p = K.Plan(_spec(num_layers=3), [2048, 777])
+    words = 3 * 8 * (2048 + 777)
+    padded = (words + 63) // 64 * 64
+    for n in (1, 2, 14):
+        assert p.select_profiles_workspace(n) == n * padded * 4
+    with pytest.raises(K.KvEvictError) as e:
+        p.select_profiles_workspace(0)
+    assert e.value.status == K.KVE_EINVAL
+    fake = ctypes.c_void_p(1 << 20)   # aligned, never dereferenced: validation fails first
+    ok = np.zeros((2, 3), np.float32)
+    for l1, l2, n in [(ok, ok, 0),
+                      (np.array([[0.5, np.nan, 0.5], [0.5, 0.5, 0.5]], np.float32), ok, 2),
+                      (ok, np.array([[0.0, 0.0, 0.0], [0.0, np.inf, 0.0]], np.float32), 2)]:
+        st = lib.kv_evict_select_profiles(p._h, n, fake, fake, fake, l1.ctypes.data, l2.ctypes.data,
+                                          fake, None, None, fake, None)
+        assert st == K.KVE_EINVAL
+    assert lib.kv_evict_select_profiles(p._h, 1, None, fake, fake, ok.ctypes.data, ok.ctypes.data,
+                                        fake, None, None, fake, None) == K.KVE_EINVAL

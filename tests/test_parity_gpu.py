@@ -131,6 +131,54 @@ def test_layer_budgets_pyramid_every_unit():
     assert torch.equal(bufs_u.k_out, bufs_p.k_out)
 
 
+@pytest.mark.parametrize("num_layers,n_prof", [(3, 5), (200, 17)])
+def test_select_profiles_equal_single_calls(num_layers, n_prof):
+    """Selection for many coefficient profiles in one pass (the search of Section 3.3
+    re-selects for every profile it tries, on the same mu and sigma): every
+    profile's indices, admission order and margins equal those of kv_evict_select
+    with that profile, bit for bit. With 200 layers one launch carries 15 profiles,
+    so 17 take two launches. One profile is also replayed through the oracle."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    seq = [700, 1300] if num_layers == 3 else [300]
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=num_layers, budget=24, seq_lens=seq)
+    batch = synth.make_batch(spec, seed=21)
+    plan, bufs, (q, k, v), _ = _run(spec, batch)
+    rng = np.random.default_rng(5)
+    l1 = rng.uniform(-1.0, 1.0, (n_prof, num_layers)).astype(np.float32)
+    l2 = rng.uniform(-1.5, 0.5, (n_prof, num_layers)).astype(np.float32)
+    l1[0] = 0.0
+    l2[0] = 0.0
+    U, B = plan.n_units, spec["budget"]
+    idx = torch.full((n_prof, U, B), -7, dtype=torch.int32, device=DEV)
+    order = torch.full_like(idx, -7)
+    mar = torch.full((n_prof, U, B), -7.0, dtype=torch.float32, device=DEV)
+    ws = torch.empty(plan.select_profiles_workspace(n_prof), dtype=torch.uint8, device=DEV)
+    plan.select_profiles(bufs.mu, bufs.sigma, k, l1, l2, idx, ws, order=order, margins=mar)
+    assert plan.status(bufs.ws) == K.KVE_OK
+    for p in range(n_prof):
+        plan.select(bufs.mu, bufs.sigma, k, l1[p], l2[p], bufs.indices, bufs.ws, order=bufs.order,
+                    margins=bufs.margins)
+        torch.cuda.synchronize()
+        assert torch.equal(idx[p], bufs.indices), p
+        assert torch.equal(order[p], bufs.order), p
+        assert torch.equal(mar[p], bufs.margins), p
+    # one profile against the oracle (a few units when there are many)
+    p = n_prof - 1
+    W, G = spec["window"], spec["num_q_heads"] // spec["num_kv_heads"]
+    units = _all_units(spec, seq) if num_layers == 3 else [(0, 0, 0), (0, 99, 3), (0, 199, 7)]
+    idx_p, ord_p, mar_p = idx[p].cpu().numpy(), order[p].cpu().numpy(), mar[p].cpu().numpy()
+    for (r, layer, h) in units:
+        L, off = seq[r], sum(seq[:r])
+        qb = PT.to_bits(batch["q_win"][layer, r, h * G:(h + 1) * G]).reshape(G * W, -1)
+        kb = PT.to_bits(batch["k"][layer, h, off:off + L])
+        kf = O.bf16_bits_to_f64(kb)
+        mu_ref, sg_ref = O.score_unit(O.bf16_bits_to_f64(qb), kf, L, W, G)
+        ui = _unit_index(spec, seq, r, layer, h)
+        PT.check_selection(ord_p[ui], idx_p[ui], mu_ref, sg_ref, kf, L, W, B, float(l1[p, layer]),
+                           float(l2[p, layer]), spec["pool_kernel"], spec["candidate_factor"],
+                           spec["norm_eps"], margins_gpu=mar_p[ui], what=f"profile {p} unit {ui}")
+
+
 @pytest.mark.parametrize("lams", [(0.0, 0.0), (0.0, -0.15), (0.5, 0.6), (-0.3, -0.5), (2.0, -3.6)])
 def test_lambda_settings(lams):
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[1200], lambdas=("global",) + lams)
