@@ -15,7 +15,8 @@
 //   phase 1 (column statistics): D[key][row] = K Q^T (keys on TMEM lanes); each
 //                               epilogue thread owns one key, forms
 //                               A = 2^(alpha*l - beta_r) for its n rows and reduces
-//                               them to mu and sigma in registers (two passes).
+//                               them to mu and sigma in registers (sums and sums of
+//                               squares; two passes where sigma/mu is small).
 // The schedule is static. CTA c owns items c, c + G, c + 2G, ... (G CTAs, all
 // resident: the launch is cooperative), so round j is items [jG, (j+1)G) and a
 // unit's items run side by side in one round (the host picks the items per unit so
@@ -107,8 +108,9 @@ struct ScoreCtl {
   uint32_t tmem_base;
   volatile int abort;
   int32_t roww[kMaxRows];                            // r % W
+  float rowm[kMaxRows];                              // 1 for rows r < n, else 0
   alignas(16) float2 comb[kItemSlots][2][kMaxRows];  // per group (m, Z) of a row item
-  alignas(16) float nbeta[kItemSlots][kMaxRows];     // -beta of a column item
+  alignas(16) float nbeta[kItemSlots][kMaxRows];     // kColScale - beta of a column item
 };
 static_assert(offsetof(ScoreCtl, nbeta) % 16 == 0, "nbeta is read with 16-byte loads");
 static_assert(offsetof(ScoreCtl, comb) % 16 == 0, "comb holds float2");
@@ -210,17 +212,27 @@ __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- epilogue, phase 1
 
-// One half (64 rows) of a key's column: A[r] = 2^(alpha*l - beta_r) for rows
-// h0..h0+63 (rows that do not see the key -- causal -- or past n give 0), the half's
-// sum and its sum of squared deviations from the half's own mean.
+// Column statistics are formed on A' = 2^kColScale * A (the staged normaliser is
+// -beta_r + kColScale): squares of A' stay normal down to A ~ 2^-103, and every sum
+// below stays far from fp32 overflow (A' <= 2^40, n <= 128).
+constexpr float kColScale = 40.f;
+constexpr float kColUnscale = 1.0f / 1099511627776.0f;   // 2^-40
+constexpr float kOnePassMin = 4e-3f;   // (sigma / mu)^2 below which the two-pass form is used
+
+// One half (64 rows) of a key's column into registers: A'[r] for rows h0..h0+63
+// (rows that do not see the key -- causal -- or past n give 0).
 template <bool kFull>
-__device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreCtl& ctl,
-                                              const float4* nb4, uint32_t taddr, int h0, int n,
-                                              int rel, float& sum, float& m2) {
+__device__ __forceinline__ void col_half_values(const ScoreParams& P, const ScoreCtl& ctl,
+                                                const float4* nb4, uint32_t taddr, int h0, int n,
+                                                int rel, float (&v)[64]) {
   const int nh = kFull ? 64 : (n - h0 < 64 ? n - h0 : 64);   // rows of this half, >= 1
-  float v[64];
   tmem_ld32(taddr + h0, v);
-  if (kFull || nh > 32) tmem_ld32(taddr + h0 + 32, v + 32);
+  if (kFull || nh > 32) {
+    tmem_ld32(taddr + h0 + 32, v + 32);
+  } else {
+#pragma unroll
+    for (int r = 32; r < 64; ++r) v[r] = 0.f;   // not loaded: rows past n
+  }
   tmem_wait_ld();
   const float2 a2 = make_float2(P.alpha, P.alpha);
 #pragma unroll
@@ -228,21 +240,65 @@ __device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreC
     const float4 b = nb4[(h0 + r) >> 2];
     const float2 x0 = ffma2(make_float2(v[r], v[r + 1]), a2, make_float2(b.x, b.y));
     const float2 x1 = ffma2(make_float2(v[r + 2], v[r + 3]), a2, make_float2(b.z, b.w));
-    v[r] = ex2(x0.x);
-    v[r + 1] = ex2(x0.y);
-    v[r + 2] = ex2(x1.x);
-    v[r + 3] = ex2(x1.y);
+    if (kFull) {
+      v[r] = ex2(x0.x);
+      v[r + 1] = ex2(x0.y);
+      v[r + 2] = ex2(x1.x);
+      v[r + 3] = ex2(x1.y);
+    } else {
+      // rows past n are staged as -inf: 2^-inf = 0 even where their products are
+      // not finite
+      v[r] = ex2(fmaxf(x0.x, -INFINITY));
+      v[r + 1] = ex2(fmaxf(x0.y, -INFINITY));
+      v[r + 2] = ex2(fmaxf(x1.x, -INFINITY));
+      v[r + 3] = ex2(fmaxf(x1.y, -INFINITY));
+    }
   }
   if (rel > 0) {
 #pragma unroll
     for (int r = 0; r < 64; ++r)
       if (rel > ctl.roww[h0 + r]) v[r] = 0.f;
   }
-  if (!kFull) {
+}
+
+// Sum and sum of squares of a half (3 fp32 operations per element with the
+// exponent's argument: the FMA pipe stays below the MUFU pipe).
+template <bool kFull>
+__device__ __forceinline__ void colsums_half(const ScoreParams& P, const ScoreCtl& ctl,
+                                             const float4* nb4, uint32_t taddr, int h0, int n,
+                                             int rel, float& sum, float& sumsq) {
+  float v[64];
+  col_half_values<kFull>(P, ctl, nb4, taddr, h0, n, rel, v);
+  float2 c0 = make_float2(0.f, 0.f), c1 = c0, c2 = c0, c3 = c0;
+  float2 q0 = c0, q1 = c0, q2 = c0, q3 = c0;
 #pragma unroll
-    for (int r = 0; r < 64; ++r)
-      if (r >= nh) v[r] = 0.f;   // rows past n (not loaded when nh <= 32)
+  for (int r = 0; r < 64; r += 8) {
+    const float2 p0 = make_float2(v[r], v[r + 1]), p1 = make_float2(v[r + 2], v[r + 3]);
+    const float2 p2 = make_float2(v[r + 4], v[r + 5]), p3 = make_float2(v[r + 6], v[r + 7]);
+    c0 = fadd2(c0, p0);
+    c1 = fadd2(c1, p1);
+    c2 = fadd2(c2, p2);
+    c3 = fadd2(c3, p3);
+    q0 = ffma2(p0, p0, q0);
+    q1 = ffma2(p1, p1, q1);
+    q2 = ffma2(p2, p2, q2);
+    q3 = ffma2(p3, p3, q3);
   }
+  const float2 cs = fadd2(fadd2(c0, c1), fadd2(c2, c3));
+  const float2 qs = fadd2(fadd2(q0, q1), fadd2(q2, q3));
+  sum = cs.x + cs.y;
+  sumsq = qs.x + qs.y;
+}
+
+// The same half, two passes: its sum and its sum of squared deviations from its own
+// mean (no cancellation; used when the one-pass form cannot be trusted).
+template <bool kFull>
+__device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreCtl& ctl,
+                                              const float4* nb4, uint32_t taddr, int h0, int n,
+                                              int rel, float& sum, float& m2) {
+  const int nh = kFull ? 64 : (n - h0 < 64 ? n - h0 : 64);
+  float v[64];
+  col_half_values<kFull>(P, ctl, nb4, taddr, h0, n, rel, v);
   float2 c0 = make_float2(0.f, 0.f), c1 = c0, c2 = c0, c3 = c0;
 #pragma unroll
   for (int r = 0; r < 64; r += 8) {
@@ -254,31 +310,14 @@ __device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreC
   const float2 cs = fadd2(fadd2(c0, c1), fadd2(c2, c3));
   sum = cs.x + cs.y;
   const float mh = sum / static_cast<float>(nh);
-  if (kFull) {
-    const float2 nm = make_float2(-mh, -mh);
-    float2 q0 = make_float2(0.f, 0.f), q1 = q0, q2 = q0, q3 = q0;
+  float q = 0.f;
 #pragma unroll
-    for (int r = 0; r < 64; r += 8) {
-      const float2 d0 = fadd2(make_float2(v[r], v[r + 1]), nm);
-      const float2 d1 = fadd2(make_float2(v[r + 2], v[r + 3]), nm);
-      const float2 d2 = fadd2(make_float2(v[r + 4], v[r + 5]), nm);
-      const float2 d3 = fadd2(make_float2(v[r + 6], v[r + 7]), nm);
-      q0 = ffma2(d0, d0, q0);
-      q1 = ffma2(d1, d1, q1);
-      q2 = ffma2(d2, d2, q2);
-      q3 = ffma2(d3, d3, q3);
-    }
-    const float2 qs = fadd2(fadd2(q0, q1), fadd2(q2, q3));
-    m2 = qs.x + qs.y;
-  } else {
-    float q = 0.f;
-#pragma unroll
-    for (int r = 0; r < 64; ++r) {
-      const float d = r < nh ? v[r] - mh : 0.f;
-      q = fmaf(d, d, q);
-    }
-    m2 = q;
+  for (int r = 0; r < 64; ++r) {
+    // rows past n: no term (ctl.rowm is 1 for rows r < n, else 0)
+    const float d = kFull ? v[r] - mh : (v[r] - mh) * ctl.rowm[h0 + r];
+    q = fmaf(d, d, q);
   }
+  m2 = q;
 }
 
 template <bool kFull>
@@ -291,6 +330,8 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
   const int n = kFull ? kMaxRows : P.g.n_rows;
   const int W = P.g.window;
   const int tile0 = d.tile0, ntiles = d.ntiles;
+  const float fn = static_cast<float>(n);
+  const float inv_n = 1.0f / fn;
   const float inv_n1 = n > 1 ? 1.0f / static_cast<float>(n - 1) : 0.f;
   const float4* nb4 = reinterpret_cast<const float4*>(ctl.nbeta[slot]);
   for (int t = 0; t < ntiles; ++t, ++ai) {
@@ -302,29 +343,46 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     const uint32_t taddr = ctl.tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + ab * 128u;
     const int key = (tile0 + t) * kTileKeys + tl;
     const int rel = key - (d.L - W);          // > 0: the key is inside the window
-    // the column's rows in two halves of 64 (registers), combined by the pairwise
-    // update of the mean and the sum of squared deviations (Chan, Golub, LeVeque)
-    float hs[2] = {0.f, 0.f}, hm2[2] = {0.f, 0.f};
+    // the column's rows in two halves of 64 (registers): one pass of sums and sums
+    // of squares, m2 = sum A'^2 - (sum A')^2 / n
     const bool two = kFull || n > 64;
+    float S1 = 0.f, SS = 0.f;
 #pragma unroll 1
     for (int h = 0; h < (two ? 2 : 1); ++h) {
-      float sh, mh2;
-      colstats_half<kFull>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, mh2);
-      if (h == 0) { hs[0] = sh; hm2[0] = mh2; } else { hs[1] = sh; hm2[1] = mh2; }
+      float sh, qh;
+      colsums_half<kFull>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, qh);
+      S1 += sh;
+      SS += qh;
     }
-    const float s1 = hs[0], m21 = hm2[0], s2 = hs[1], m22 = hm2[1];
+    float m2 = fmaf(-S1, S1 * inv_n, SS);
+    // The one-pass form loses about (sum A'^2) * 2^-19 to rounding. It is kept while
+    // sigma^2 >= kOnePassMin * mu^2, where that loss stays below 2e-4 of sigma^2;
+    // otherwise (columns of nearly equal A, e.g. uniform attention) the warp takes
+    // the two-pass form over the same TMEM columns, halves combined by the pairwise
+    // update of the mean and the sum of squared deviations (Chan, Golub, LeVeque).
+    const bool exact = !(m2 * fn * fn >= kOnePassMin * (fn - 1.f) * S1 * S1);   // NaN-safe
+    if (__any_sync(0xffffffffu, exact)) {
+      float hs[2] = {0.f, 0.f}, hm2[2] = {0.f, 0.f};
+#pragma unroll 1
+      for (int h = 0; h < (two ? 2 : 1); ++h) {
+        float sh, mh2;
+        colstats_half<kFull>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, mh2);
+        if (h == 0) { hs[0] = sh; hm2[0] = mh2; } else { hs[1] = sh; hm2[1] = mh2; }
+      }
+      const float n1 = kFull ? 64.f : static_cast<float>(n < 64 ? n : 64);
+      const float n2 = fn - n1;
+      float m2x = hm2[0] + hm2[1];
+      if (two) {
+        const float dd = hs[1] / n2 - hs[0] / n1;
+        m2x = fmaf(dd * dd, n1 * n2 * inv_n, m2x);
+      }
+      if (exact) m2 = m2x;
+    }
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(&ctl.acc_empty[ab]);
-    const float n1 = kFull ? 64.f : static_cast<float>(n < 64 ? n : 64);
-    const float n2 = static_cast<float>(n) - n1;
-    const float mu = (s1 + s2) / static_cast<float>(n);
-    float m2 = m21 + m22;
-    if (two) {
-      const float d = s2 / n2 - s1 / n1;
-      m2 = fmaf(d * d, n1 * n2 / static_cast<float>(n), m2);
-    }
-    const float sigma = sqrtf(fmaxf(m2, 0.f) * inv_n1);
+    const float mu = S1 * inv_n * kColUnscale;
+    const float sigma = sqrtf(fmaxf(m2, 0.f) * inv_n1) * kColUnscale;
     if (key < d.L) {
       __stcs(&P.mu[d.mu_off + key], mu);
       __stcs(&P.sigma[d.mu_off + key], sigma);
@@ -355,10 +413,10 @@ __device__ __forceinline__ bool stage_beta(const ScoreParams& P, ScoreCtl& ctl,
   for (int k = 0; k < 4; ++k) ready = ready && (w[k] >> 32) != 0ull;
   if (!__all_sync(0xffffffffu, ready)) return false;
   float4 b;
-  b.x = r0 + 0 < n ? -__uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
-  b.y = r0 + 1 < n ? -__uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
-  b.z = r0 + 2 < n ? -__uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
-  b.w = r0 + 3 < n ? -__uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
+  b.x = r0 + 0 < n ? kColScale - __uint_as_float(static_cast<uint32_t>(w[0])) : -INFINITY;
+  b.y = r0 + 1 < n ? kColScale - __uint_as_float(static_cast<uint32_t>(w[1])) : -INFINITY;
+  b.z = r0 + 2 < n ? kColScale - __uint_as_float(static_cast<uint32_t>(w[2])) : -INFINITY;
+  b.w = r0 + 3 < n ? kColScale - __uint_as_float(static_cast<uint32_t>(w[3])) : -INFINITY;
   reinterpret_cast<float4*>(ctl.nbeta[slot])[lane] = b;
   return true;
 }
@@ -538,7 +596,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tensormap(&tm_q);
     prefetch_tensormap(&tm_k);
   }
-  if (threadIdx.x < kMaxRows) ctl.roww[threadIdx.x] = threadIdx.x % P.g.window;
+  if (threadIdx.x < kMaxRows) {
+    ctl.roww[threadIdx.x] = threadIdx.x % P.g.window;
+    ctl.rowm[threadIdx.x] = static_cast<int>(threadIdx.x) < P.g.n_rows ? 1.f : 0.f;
+  }
   if (warp == 1) {
     tmem_alloc(&ctl.tmem_base, kTmemCols);
     tmem_relinquish();
