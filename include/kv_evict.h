@@ -104,6 +104,24 @@ kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens,
                                  int32_t n_req, const int32_t* layer_budgets,
                                  kve_plan** plan_out, size_t* workspace_bytes);
 
+/* Flags of kv_evict_plan_ex. */
+#define KVE_PLAN_PER_QUERY_HEAD 1
+
+/* kv_evict_plan_layered with flags (0 = kv_evict_plan_layered).
+ * KVE_PLAN_PER_QUERY_HEAD: every query head selects its own tokens. The paper leaves
+ * the GQA grouping open; the default pools the G*W window rows of the query heads
+ * that share a KV head into one unit (n = G*W rows, one selection per KV head).
+ * With this flag a unit is (request, layer, query head): its n = W rows are that
+ * head's window queries, its keys those of its KV head (query head hq reads KV head
+ * hq / G), and the selection, the compact cache and every per-unit array are
+ * indexed by query head: mu, sigma [n_req][N_L][Hq][L_r]; indices, order, margins
+ * [n_req][N_L][Hq][B]; k_out, v_out [n_req][N_L][Hq][B+W][d]. Inputs keep their
+ * layouts. Other flag bits: KVE_EINVAL. */
+kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens,
+                            int32_t n_req, const int32_t* layer_budgets,
+                            int32_t flags, kve_plan** plan_out,
+                            size_t* workspace_bytes);
+
 void kv_evict_plan_destroy(kve_plan* plan);
 
 /* Test hook: limit (ns) of every device-side bounded wait of later calls with this

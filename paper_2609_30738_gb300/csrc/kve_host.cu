@@ -81,7 +81,7 @@ int32_t choose_splits(int64_t T, int64_t ctas) {
 // width) stay in L2 for the phase-1 re-read.
 int32_t score_lag(const kve::Geometry& g, int64_t ctas) {
   int64_t span = 0;
-  const int64_t units_per_req = static_cast<int64_t>(g.num_layers) * g.hkv;
+  const int64_t units_per_req = static_cast<int64_t>(g.num_layers) * g.uheads;
   for (int r = 0; r < g.n_req; ++r) {
     const int64_t k = g.req_splits[r];
     // (first item) mod ctas repeats with period ctas / gcd(k, ctas) <= ctas
@@ -106,7 +106,14 @@ kve_status kv_evict_plan(const kve_config* cfg, const int64_t* seq_lens, int32_t
 kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens, int32_t n_req,
                                  const int32_t* layer_budgets, kve_plan** plan_out,
                                  size_t* workspace_bytes) {
+  return kv_evict_plan_ex(cfg, seq_lens, n_req, layer_budgets, 0, plan_out, workspace_bytes);
+}
+
+kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens, int32_t n_req,
+                            const int32_t* layer_budgets, int32_t flags, kve_plan** plan_out,
+                            size_t* workspace_bytes) {
   if (!cfg || !seq_lens || !plan_out) return KVE_EINVAL;
+  if ((flags & ~KVE_PLAN_PER_QUERY_HEAD) != 0) return KVE_EINVAL;
   *plan_out = nullptr;
   const kve_config& c = *cfg;
   if (c.num_layers < 1 || c.num_layers > kMaxLayers) return KVE_EINVAL;
@@ -140,9 +147,12 @@ kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens,
   g.hkv = c.num_kv_heads;
   g.group = G;
   g.window = c.window;
-  g.n_rows = G * c.window;
+  const bool per_q = (flags & KVE_PLAN_PER_QUERY_HEAD) != 0;
+  g.uheads = per_q ? c.num_q_heads : c.num_kv_heads;
+  g.ugroup = per_q ? 1 : G;
+  g.n_rows = g.ugroup * c.window;
   int64_t off = 0, units = 0, items = 0, max_lc = 0;
-  const int64_t units_per_req = static_cast<int64_t>(c.num_layers) * c.num_kv_heads;
+  const int64_t units_per_req = static_cast<int64_t>(c.num_layers) * g.uheads;
   int ctas = device_sms();
   if (ctas <= 0) {
     cudaGetLastError();
@@ -173,7 +183,7 @@ kve_status kv_evict_plan_layered(const kve_config* cfg, const int64_t* seq_lens,
   const int64_t max_cand = c.candidate_factor == 0 ? max_lc
                                                    : std::min<int64_t>(int64_t(c.candidate_factor) * c.budget, max_lc);
   // TMA row coordinates are 32-bit; the select kernel holds its pool in shared memory
-  const int64_t k_rows = units_per_req * off;
+  const int64_t k_rows = static_cast<int64_t>(c.num_layers) * c.num_kv_heads * off;
   const int64_t q_rows = static_cast<int64_t>(c.num_layers) * n_req * c.num_q_heads * c.window;
   if (max_cand > kMaxCand || k_rows >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
       2 * items >= (int64_t(1) << 31) || units >= (int64_t(1) << 31)) {
@@ -270,7 +280,7 @@ kve_status select_params(const kve_plan* plan, const float* mu, const float* sig
 // every unit), padded to 256 bytes.
 int64_t profile_keys_words(const kve_plan* plan) {
   const kve::Geometry& g = plan->geo;
-  const int64_t words = static_cast<int64_t>(g.num_layers) * g.hkv * g.total_tokens;
+  const int64_t words = static_cast<int64_t>(g.num_layers) * g.uheads * g.total_tokens;
   return (words + 63) / 64 * 64;
 }
 

@@ -21,8 +21,11 @@ constexpr int kMaxLayers = 256;    // layers per call (lambda arrays ride in ker
 // Request table and derived counts, identical on host and device.
 struct Geometry {
   int32_t n_req, num_layers, hq, hkv, group, window, n_rows;
+  int32_t uheads;                       // heads per layer that own a unit: hkv, or hq
+                                        // when every query head selects for itself
+  int32_t ugroup;                       // query heads per unit: group, or 1
   int64_t total_tokens;                 // SL
-  int64_t n_units;                      // n_req * N_L * Hkv
+  int64_t n_units;                      // n_req * N_L * uheads
   int64_t n_items;                      // score work items (sum over units of splits)
   int32_t req_len[kMaxReq];             // L_r
   int64_t req_tok_off[kMaxReq];         // off_r
@@ -52,16 +55,17 @@ __host__ __device__ inline UnitInfo unit_info(const Geometry& g, int64_t unit) {
   u.unit = unit;
   u.r = r;
   const int64_t local = unit - g.req_unit_base[r];
-  u.layer = static_cast<int32_t>(local / g.hkv);
-  u.h = static_cast<int32_t>(local % g.hkv);
+  u.layer = static_cast<int32_t>(local / g.uheads);
+  u.h = static_cast<int32_t>(local % g.uheads);   // KV head (or query head) of the unit
   u.L = g.req_len[r];
   u.tiles = g.req_tiles[r];
   u.splits = g.req_splits[r];
   u.local = local;
   u.q_row0 = ((static_cast<int64_t>(u.layer) * g.n_req + r) * g.hq +
-              static_cast<int64_t>(u.h) * g.group) * g.window;
-  u.k_row0 = (static_cast<int64_t>(u.layer) * g.hkv + u.h) * g.total_tokens + g.req_tok_off[r];
-  u.mu_off = static_cast<int64_t>(g.num_layers) * g.hkv * g.req_tok_off[r] + local * u.L;
+              static_cast<int64_t>(u.h) * g.ugroup) * g.window;
+  const int kvh = g.ugroup == g.group ? u.h : u.h / g.group;   // the KV head the unit reads
+  u.k_row0 = (static_cast<int64_t>(u.layer) * g.hkv + kvh) * g.total_tokens + g.req_tok_off[r];
+  u.mu_off = static_cast<int64_t>(g.num_layers) * g.uheads * g.req_tok_off[r] + local * u.L;
   u.item0 = g.req_item_base[r] + local * u.splits;
   return u;
 }

@@ -591,7 +591,7 @@ extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float*
   using namespace kve;
   if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices) return KVE_EINVAL;
   const Geometry& g = plan->geo;
-  const size_t words = static_cast<size_t>(g.num_layers) * g.hkv * static_cast<size_t>(g.total_tokens);
+  const size_t words = static_cast<size_t>(g.num_layers) * g.uheads * static_cast<size_t>(g.total_tokens);
   if (words > kNoAllocScratchWords) return KVE_EINVAL;   // beyond the fixed scratch
   if ((reinterpret_cast<uintptr_t>(k) & 15u) != 0) return KVE_EINVAL;
   uint32_t* scratch = scratch_on_current_device();

@@ -18,7 +18,8 @@ LIB_PATH = os.path.join(_HERE, "libkvevict.so")
 KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 
 # Names declared in include/kv_evict.h.
-EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_destroy", "kv_evict_plan_set_debug",
+EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_destroy",
+           "kv_evict_plan_set_debug",
            "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
            "kv_evict_select_profiles_workspace", "kv_evict_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
@@ -53,6 +54,8 @@ def _lib():
                                       ctypes.POINTER(vp), ctypes.POINTER(ctypes.c_size_t)]
         lib.kv_evict_plan_layered.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32, vp,
                                               ctypes.POINTER(vp), ctypes.POINTER(ctypes.c_size_t)]
+        lib.kv_evict_plan_ex.argtypes = [ctypes.POINTER(Config), ctypes.POINTER(i64), i32, vp, i32,
+                                         vp, vp]
         lib.kv_evict_budget_pyramid.argtypes = [i32, i32, ctypes.c_float, vp]
         lib.kv_evict_plan_destroy.argtypes = [vp]
         lib.kv_evict_plan_destroy.restype = None
@@ -67,7 +70,7 @@ def _lib():
         lib.kv_evict_profile.argtypes = [i32, vp, i32, vp, vp]
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
         lib.kv_evict_strerror.restype = ctypes.c_char_p
-        for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_set_debug",
+        for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_set_debug",
                      "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc",
                      "kv_evict_select_profiles", "kv_evict_select_profiles_workspace", "kv_evict_gather",
                      "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
@@ -109,11 +112,15 @@ def make_config(spec: dict) -> Config:
                   spec.get("candidate_factor", 4), spec.get("norm_eps", 1e-12))
 
 
+KVE_PLAN_PER_QUERY_HEAD = 1
+
+
 class Plan:
-    """kv_evict_plan (kv_evict_plan_layered when layer_budgets is given) for a
+    """kv_evict_plan (kv_evict_plan_layered when layer_budgets is given,
+    kv_evict_plan_ex with KVE_PLAN_PER_QUERY_HEAD when per_query_head) for a
     configuration and the prefix lengths of the requests."""
 
-    def __init__(self, spec: dict, seq_lens, layer_budgets=None):
+    def __init__(self, spec: dict, seq_lens, layer_budgets=None, per_query_head: bool = False):
         lib = _lib()
         self.spec = dict(spec)
         self.seq_lens = [int(x) for x in seq_lens]
@@ -121,7 +128,15 @@ class Plan:
         lens = (ctypes.c_int64 * len(self.seq_lens))(*self.seq_lens)
         handle = ctypes.c_void_p()
         ws = ctypes.c_size_t()
-        if layer_budgets is None:
+        self.per_query_head = bool(per_query_head)
+        if self.per_query_head:
+            self.layer_budgets = ([int(spec["budget"])] * int(spec["num_layers"]) if layer_budgets is None
+                                  else [int(b) for b in layer_budgets])
+            lb = np.ascontiguousarray(self.layer_budgets, dtype=np.int32)
+            _check(lib.kv_evict_plan_ex(ctypes.byref(self._cfg), lens, len(self.seq_lens), lb.ctypes.data,
+                                        KVE_PLAN_PER_QUERY_HEAD, ctypes.byref(handle), ctypes.byref(ws)),
+                   "kv_evict_plan_ex")
+        elif layer_budgets is None:
             self.layer_budgets = [int(spec["budget"])] * int(spec["num_layers"])
             _check(lib.kv_evict_plan(ctypes.byref(self._cfg), lens, len(self.seq_lens),
                                      ctypes.byref(handle), ctypes.byref(ws)), "kv_evict_plan")
@@ -142,12 +157,17 @@ class Plan:
 
     # -- sizes of the documented layouts
     @property
+    def unit_heads(self) -> int:
+        """Heads per layer that own a unit: KV heads, or query heads per_query_head."""
+        return self.spec["num_q_heads"] if self.per_query_head else self.spec["num_kv_heads"]
+
+    @property
     def n_units(self) -> int:
-        return len(self.seq_lens) * self.spec["num_layers"] * self.spec["num_kv_heads"]
+        return len(self.seq_lens) * self.spec["num_layers"] * self.unit_heads
 
     @property
     def score_elems(self) -> int:
-        return self.spec["num_layers"] * self.spec["num_kv_heads"] * sum(self.seq_lens)
+        return self.spec["num_layers"] * self.unit_heads * sum(self.seq_lens)
 
     def set_debug(self, wait_limit_ns: int, fault: int = 0):
         _check(_lib().kv_evict_plan_set_debug(self._h, int(wait_limit_ns), int(fault)),

@@ -145,3 +145,26 @@ def test_select_profiles_validation_without_gpu():
         assert st == K.KVE_EINVAL
     assert lib.kv_evict_select_profiles(p._h, 1, None, fake, fake, ok.ctypes.data, ok.ctypes.data,
                                         fake, None, None, fake, None) == K.KVE_EINVAL
+
+
+def test_plan_ex_flags_without_gpu():
+    """kv_evict_plan_ex: flag 0 is the layered plan, KVE_PLAN_PER_QUERY_HEAD makes one
+    unit per query head, other bits are rejected."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = _spec(num_layers=3)
+    base = K.Plan(spec, [2048, 777])
+    perq = K.Plan(spec, [2048, 777], per_query_head=True)
+    assert perq.n_units == 2 * 3 * 32 and base.n_units == 2 * 3 * 8
+    assert perq.score_elems == 3 * 32 * (2048 + 777)
+    assert perq.workspace_bytes > base.workspace_bytes
+    lib = K.library()
+    cfg = K.make_config(spec)
+    lens = (ctypes.c_int64 * 1)(500)
+    h, ws = ctypes.c_void_p(), ctypes.c_size_t()
+    for bad in (2, 4, -1):
+        assert lib.kv_evict_plan_ex(ctypes.byref(cfg), lens, 1, None, bad, ctypes.byref(h),
+                                    ctypes.byref(ws)) == K.KVE_EINVAL
+    assert lib.kv_evict_plan_ex(ctypes.byref(cfg), lens, 1, None, 0, ctypes.byref(h),
+                                ctypes.byref(ws)) == K.KVE_OK
+    lib.kv_evict_plan_destroy(h)

@@ -131,6 +131,68 @@ def test_layer_budgets_pyramid_every_unit():
     assert torch.equal(bufs_u.k_out, bufs_p.k_out)
 
 
+def test_per_query_head_selection_every_unit():
+    """Every query head selects for itself (the alternative GQA reading): unit
+    (request, layer, query head) with its own W window rows (n = W) against the
+    keys of its KV head, checked against the oracle run on exactly those rows."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=24, seq_lens=[900, 1400])
+    batch = synth.make_batch(spec, seed=41)
+    seq = batch["seq_lens"]
+    plan = K.Plan(spec, seq, per_query_head=True)
+    assert plan.n_units == 2 * 2 * spec["num_q_heads"]
+    bufs = K.Buffers(plan)
+    lam = lambda_arrays(spec, K.profile)
+    q, k, v = (batch[x].to(DEV) for x in ("q_win", "k", "v"))
+    K.run_step(plan, bufs, q, k, v, lam[0], lam[1])
+    assert plan.status(bufs.ws) == K.KVE_OK
+    W, B, Hq, G = spec["window"], spec["budget"], spec["num_q_heads"], spec["num_q_heads"] // spec["num_kv_heads"]
+    N_L = spec["num_layers"]
+    mu_all, sg_all = bufs.mu.cpu().numpy(), bufs.sigma.cpu().numpy()
+    idx_all, ord_all, mar_all = (bufs.indices.cpu().numpy(), bufs.order.cpu().numpy(),
+                                 bufs.margins.cpu().numpy())
+    for r in range(len(seq)):
+        L, off = seq[r], sum(seq[:r])
+        for layer in range(N_L):
+            for hq in range(Hq):
+                kvh = hq // G
+                qb = PT.to_bits(batch["q_win"][layer, r, hq]).reshape(W, -1)
+                kb = PT.to_bits(batch["k"][layer, kvh, off:off + L])
+                vb = PT.to_bits(batch["v"][layer, kvh, off:off + L])
+                kf = O.bf16_bits_to_f64(kb)
+                mu_ref, sg_ref = O.score_unit(O.bf16_bits_to_f64(qb), kf, L, W, 1)
+                ui = (r * N_L + layer) * Hq + hq
+                o = N_L * Hq * sum(seq[:r]) + (layer * Hq + hq) * L
+                tag = f"unit(r={r},l={layer},hq={hq})"
+                PT.check_mu_sigma(mu_all[o:o + L], sg_all[o:o + L], mu_ref, sg_ref, tag)
+                PT.check_selection(ord_all[ui], idx_all[ui], mu_ref, sg_ref, kf, L, W, B,
+                                   float(lam[0][layer]), float(lam[1][layer]), spec["pool_kernel"],
+                                   spec["candidate_factor"], spec["norm_eps"], margins_gpu=mar_all[ui],
+                                   what=tag)
+                PT.check_gather(PT.to_bits(bufs.k_out[ui]), PT.to_bits(bufs.v_out[ui]), kb, vb,
+                                idx_all[ui], L, W, B)
+
+
+def test_per_query_head_equals_default_without_grouping():
+    """With one query head per KV head (G = 1) both readings define the same units:
+    the per-query-head plan gives the default plan's outputs bit for bit."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_q_heads=8, window=64, budget=16,
+                  seq_lens=[1000, 333])
+    batch = synth.make_batch(spec, seed=43)
+    outs = []
+    for per_q in (False, True):
+        plan = K.Plan(spec, batch["seq_lens"], per_query_head=per_q)
+        bufs = K.Buffers(plan)
+        lam = lambda_arrays(spec, K.profile)
+        q, k, v = (batch[x].to(DEV) for x in ("q_win", "k", "v"))
+        K.run_step(plan, bufs, q, k, v, lam[0], lam[1])
+        assert plan.status(bufs.ws) == K.KVE_OK
+        outs.append((bufs.mu.clone(), bufs.sigma.clone(), bufs.indices.clone(), bufs.k_out.clone()))
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
 @pytest.mark.parametrize("num_layers,n_prof", [(3, 5), (200, 17)])
 def test_select_profiles_equal_single_calls(num_layers, n_prof):
     """Selection for many coefficient profiles in one pass (the search of Section 3.3
