@@ -15,7 +15,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libkvevict.so")
-SOURCES = ["kve_host.cu", "kve_score.cu", "kve_select.cu", "kve_gather.cu"]
+SOURCES = ["kve_host.cu", "kve_score.cu", "kve_select.cu", "kve_select_all.cu", "kve_gather.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xptxas", "-v"]

@@ -21,7 +21,6 @@ using kve::kSplitTiles;
 using kve::kTileKeys;
 
 constexpr uint64_t kDefaultWaitNs = 2000000000ull;   // 2 s
-constexpr int kMaxCand = 512;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -185,7 +184,12 @@ kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens, int3
   // TMA row coordinates are 32-bit; the select kernel holds its pool in shared memory
   const int64_t k_rows = static_cast<int64_t>(c.num_layers) * c.num_kv_heads * off;
   const int64_t q_rows = static_cast<int64_t>(c.num_layers) * n_req * c.num_q_heads * c.window;
-  if (max_cand > kMaxCand || k_rows >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
+  // candidate_factor = 0 beyond the pooled selector's pool runs the every-candidate
+  // selector (Lc <= kMaxAllCand, B <= kMaxAllBudget)
+  plan->select_all = (c.candidate_factor == 0 && max_lc > kve::kMaxPoolCand) ? 1 : 0;
+  const bool cand_ok = plan->select_all ? (max_lc <= kve::kMaxAllCand && c.budget <= kve::kMaxAllBudget)
+                                        : max_cand <= kve::kMaxPoolCand;
+  if (!cand_ok || k_rows >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
       2 * items >= (int64_t(1) << 31) || units >= (int64_t(1) << 31)) {
     delete plan;
     return KVE_EINVAL;
@@ -197,7 +201,9 @@ kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens, int3
   w.clear_end = align_up(w.beta + sizeof(uint64_t) * kMaxRows * units, 256);
   w.partial = w.clear_end;
   w.keys = align_up(w.partial + sizeof(float2) * kMaxRows * items, 256);
-  w.total = align_up(w.keys + sizeof(uint32_t) * units_per_req * off, 256);
+  w.corr = plan->select_all ? align_up(w.keys + sizeof(uint32_t) * units_per_req * off, 256) : 0;
+  w.total = plan->select_all ? align_up(w.corr + sizeof(float2) * units_per_req * off, 256)
+                              : align_up(w.keys + sizeof(uint32_t) * units_per_req * off, 256);
   if (workspace_bytes) *workspace_bytes = w.total;
   *plan_out = plan;
   return KVE_OK;
@@ -302,11 +308,16 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
   const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
   if (s != KVE_OK) return s;
   p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.keys);
+  if (plan->select_all) {
+    p.corr = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + plan->ws.corr);
+    return kve::launch_select_all(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK
+                                                                                              : KVE_ECUDA;
+  }
   return kve::launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
 }
 
 kve_status kv_evict_select_profiles_workspace(const kve_plan* plan, int32_t n_profiles, size_t* bytes) {
-  if (!plan || !bytes || n_profiles < 1) return KVE_EINVAL;
+  if (!plan || !bytes || n_profiles < 1 || plan->select_all) return KVE_EINVAL;
   *bytes = static_cast<size_t>(n_profiles) * static_cast<size_t>(profile_keys_words(plan)) * sizeof(uint32_t);
   return KVE_OK;
 }
@@ -315,7 +326,8 @@ kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles, co
                                     const float* sigma, const uint16_t* k, const float* lambda1,
                                     const float* lambda2, int32_t* indices, int32_t* order, float* margins,
                                     void* ws, void* stream) {
-  if (!plan || n_profiles < 1 || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws)
+  if (!plan || n_profiles < 1 || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws ||
+      plan->select_all)
     return KVE_EINVAL;
   if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
   const int32_t nl = plan->geo.num_layers;

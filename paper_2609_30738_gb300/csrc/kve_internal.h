@@ -17,6 +17,9 @@ constexpr int kSplitTiles = 8;     // most tiles in one work item
 constexpr int kMaxRows = 128;      // n = G*W window rows per unit, padded to one M tile
 constexpr int kMaxReq = 64;        // requests per call
 constexpr int kMaxLayers = 256;    // layers per call (lambda arrays ride in kernel params)
+constexpr int kMaxPoolCand = 512;  // candidate pool of the pooled selector (shared memory)
+constexpr int kMaxAllCand = 32768; // candidates of the every-candidate selector (Lc)
+constexpr int kMaxAllBudget = 1024;// admissions of the every-candidate selector
 
 // Request table and derived counts, identical on host and device.
 struct Geometry {
@@ -98,6 +101,7 @@ struct WsLayout {
   size_t clear_end;  // bytes from 0 cleared before each score call
   size_t partial;    // float2 [n_items][kMaxRows]  per-item (max, sum) in log2 units
   size_t keys;       // uint32 [sum of unit lengths]  ordered base scores (select)
+  size_t corr;       // float2 [sum of unit lengths]  (corr, 1/|k|): every-candidate selector only
   size_t total;
 };
 
@@ -127,6 +131,8 @@ struct SelectParams {
   int32_t* order;
   float* margins;
   uint32_t* keys;            // workspace scratch
+  float* corr;               // workspace scratch of the every-candidate selector (or null):
+                             // float2 (corr, 1/|k|) per prefix token of every unit
   float lambda1[kMaxLayers];
   float lambda2[kMaxLayers];
   int32_t layer_budget[kMaxLayers];   // B_l <= budget kept candidates of layer l
@@ -166,6 +172,8 @@ struct kve_plan {
   kve::WsLayout ws;
   uint64_t wait_limit_ns;
   int32_t fault;
+  int32_t select_all;   // 1: candidate_factor = 0 and some Lc exceeds kMaxPoolCand, so the
+                        // selection runs on the every-candidate selector
 };
 
 namespace kve {
@@ -173,6 +181,7 @@ namespace kve {
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                          const ScoreParams& p, int ctas, cudaStream_t stream);
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
+cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_select_profiles(const kve_plan& plan, const SelectParams& p, const ProfileTable& table,
                                    int profiles, cudaStream_t stream);
 cudaError_t launch_gather(const kve_plan& plan, const GatherParams& p, cudaStream_t stream);

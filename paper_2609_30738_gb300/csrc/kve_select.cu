@@ -589,7 +589,8 @@ extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float*
                                               const float* lambda2, int32_t* indices, int32_t* order,
                                               float* margins, void* stream) {
   using namespace kve;
-  if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices) return KVE_EINVAL;
+  if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || plan->select_all)
+    return KVE_EINVAL;
   const Geometry& g = plan->geo;
   const size_t words = static_cast<size_t>(g.num_layers) * g.uheads * static_cast<size_t>(g.total_tokens);
   if (words > kNoAllocScratchWords) return KVE_EINVAL;   // beyond the fixed scratch

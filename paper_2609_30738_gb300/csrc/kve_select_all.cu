@@ -1,0 +1,269 @@
+// Selector over every candidate (candidate_factor = 0 with Lc above the pooled
+// selector's 512-slot pool): step 3 of the eviction step with C = Lc, one CTA per
+// unit. Section 3.2 restricts the greedy to the top 4B tokens for speed; this path
+// is the unrestricted ablation and admits exactly what the full greedy of Eq. 5
+// admits over all Lc candidates.
+//
+//  1. max-pool mu and sigma over 0 .. Lc-1 (odd kernel, window clipped to the
+//     range) and form s_i = mu_i + lambda1 sigma_i; s~ = s / max(max s, eps);
+//  2. greedy admissions by s~_i + lambda2 corr_i, ties to the lower position, with
+//     corr_i = max over admitted j of cos(k_i, k_j) (clamped at 0 by starting at 0).
+//     With lambda2 <= 0 a value can only fall as the admitted set grows, so a value
+//     computed against fewer admitted keys is an upper bound: each step takes the
+//     best value; if it is stale, every thread whose own best candidate is stale
+//     brings that candidate up to date (in parallel) and the search repeats; a
+//     candidate whose value is current when it is the best is the full greedy's
+//     choice (any candidate with an equal bound has a higher position).
+//     With lambda2 > 0 every candidate is brought up to date after each admission.
+//     When margins are requested the runner-up is brought up to date the same way.
+//  3. write the admitted positions ascending (and in admission order, with margins).
+// Values live in shared memory (C <= 32768); s~, corr and the inverse key norms in
+// the workspace; the admitted keys are read from K in global memory (L2).
+#include "kve_internal.h"
+
+namespace kve {
+namespace {
+
+constexpr int kAllThreads = 1024;
+constexpr int kAllWarps = kAllThreads / 32;
+
+__device__ __forceinline__ uint32_t ord_key_all(float f) {
+  const uint32_t u = __float_as_uint(f + 0.0f);   // -0 -> +0
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+struct AllSmall {
+  uint32_t wkey[kAllWarps];
+  uint32_t widx[kAllWarps];
+  float wmax[kAllWarps];
+  uint32_t best_key, best_idx;
+  int32_t refreshed;
+};
+
+// Block argmax of the owners' bests: the largest key, ties to the lowest index.
+__device__ __forceinline__ void block_best(uint32_t key, uint32_t idx, AllSmall& sh) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t wk = __reduce_max_sync(0xffffffffu, key);
+  const uint32_t wi = __reduce_min_sync(0xffffffffu, key == wk ? idx : 0xFFFFFFFFu);
+  if (lane == 0) {
+    sh.wkey[warp] = wk;
+    sh.widx[warp] = wi;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t k = sh.wkey[lane], i = sh.widx[lane];
+    const uint32_t bk = __reduce_max_sync(0xffffffffu, k);
+    const uint32_t bi = __reduce_min_sync(0xffffffffu, k == bk ? i : 0xFFFFFFFFu);
+    if (lane == 0) {
+      sh.best_key = bk;
+      sh.best_idx = bi;
+    }
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid_constant__ SelectParams P) {
+  __shared__ AllSmall sh;
+  extern __shared__ __align__(16) uint8_t dyn[];
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+
+  const UnitInfo u = unit_info(P.g, blockIdx.x);
+  const int W = P.g.window;
+  const int C = u.L - W;                      // every candidate
+  const int B = P.budget;
+  const int Bl = P.layer_budget[u.layer];
+  const int nsel = min(Bl, C);
+  const float lambda1 = P.lambda1[u.layer];
+  const float lambda2 = P.lambda2[u.layer];
+  const bool lazy = !(lambda2 > 0.f);
+  const float* mu = P.mu + u.mu_off;
+  const float* sg = P.sigma + u.mu_off;
+  float* st = reinterpret_cast<float*>(P.keys + u.mu_off);   // s~ per candidate
+  float2* cinv = reinterpret_cast<float2*>(P.corr) + u.mu_off;   // (corr_i, 1 / |k_i|)
+  const uint16_t* kb = P.k + u.k_row0 * kHeadDim;
+  const int h = P.pool_kernel / 2;
+
+  float* v = reinterpret_cast<float*>(dyn);                         // [kMaxAllCand]
+  uint16_t* applied = reinterpret_cast<uint16_t*>(v + kMaxAllCand);  // [kMaxAllCand]
+  int32_t* adm = reinterpret_cast<int32_t*>(applied + kMaxAllCand);  // [kMaxAllBudget]
+  float* adm_inv = reinterpret_cast<float*>(adm + kMaxAllBudget);    // [kMaxAllBudget]
+
+  // 1. pooled base score and its maximum
+  float lmax = -INFINITY;
+  for (int i = tid; i < C; i += kAllThreads) {
+    const int a = max(i - h, 0), b = min(i + h, C - 1);
+    float mh = -INFINITY, shh = -INFINITY;
+    for (int j = a; j <= b; ++j) {
+      mh = fmaxf(mh, __ldg(mu + j));
+      shh = fmaxf(shh, __ldg(sg + j));
+    }
+    const float s = fmaf(lambda1, shh, mh);
+    st[i] = s;
+    lmax = fmaxf(lmax, s);
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, o));
+  if (lane == 0) sh.wmax[warp] = lmax;
+  __syncthreads();
+  float smax = sh.wmax[0];
+  for (int w = 1; w < kAllWarps; ++w) smax = fmaxf(smax, sh.wmax[w]);
+  smax = fmaxf(smax, P.norm_eps);
+  for (int i = tid; i < C; i += kAllThreads) {
+    const float s = __fdiv_rn(st[i], smax);
+    st[i] = s;
+    v[i] = s;                     // corr = 0: s~ + lambda2 * 0
+    applied[i] = 0;
+    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kHeadDim);
+    float ss = 0.f;
+    for (int c = 0; c < kHeadDim / 8; ++c) {
+      const uint4 x = __ldg(ki + c);
+      const uint32_t w4[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        ss = fmaf(bf16_lo(w4[e]), bf16_lo(w4[e]), ss);
+        ss = fmaf(bf16_hi(w4[e]), bf16_hi(w4[e]), ss);
+      }
+    }
+    cinv[i] = make_float2(0.f, ss > 0.f ? __fdiv_rn(1.0f, sqrtf(ss)) : 0.f);
+  }
+  __syncthreads();
+
+  // the owner of candidate i is thread i % kAllThreads; it keeps the best of its own
+  uint32_t my_key = 0, my_idx = 0xFFFFFFFFu;
+  auto rescan = [&]() {
+    my_key = 0;
+    my_idx = 0xFFFFFFFFu;
+    for (int i = tid; i < C; i += kAllThreads) {
+      const float x = v[i];
+      if (x == -INFINITY) continue;   // admitted
+      const uint32_t k = ord_key_all(x);
+      if (k > my_key || my_idx == 0xFFFFFFFFu) {
+        my_key = k;
+        my_idx = static_cast<uint32_t>(i);
+      }
+    }
+  };
+  rescan();
+
+  // candidate i brought up to date with admissions applied[i] .. t-1 by its owner
+  auto refresh = [&](int i, int t) {
+    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kHeadDim);
+    const float2 ci = cinv[i];
+    const float inv_i = ci.y;
+    float cmax = ci.x;
+    for (int a = applied[i]; a < t; ++a) {
+      const uint4* kj = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(adm[a]) * kHeadDim);
+      float dot = 0.f;
+      for (int c = 0; c < kHeadDim / 8; ++c) {
+        const uint4 x = __ldg(ki + c), y = __ldg(kj + c);
+        const uint32_t xa[4] = {x.x, x.y, x.z, x.w}, ya[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          dot = fmaf(bf16_lo(xa[e]), bf16_lo(ya[e]), dot);
+          dot = fmaf(bf16_hi(xa[e]), bf16_hi(ya[e]), dot);
+        }
+      }
+      cmax = fmaxf(cmax, dot * inv_i * adm_inv[a]);
+    }
+    cinv[i] = make_float2(cmax, inv_i);
+    v[i] = fmaf(lambda2, cmax, st[i]);
+    applied[i] = static_cast<uint16_t>(t);
+  };
+  // every owner whose best is stale brings it up to date, then takes its new best
+  auto refresh_stale_bests = [&](int t) {
+    if (my_idx != 0xFFFFFFFFu && applied[my_idx] < t) {
+      refresh(static_cast<int>(my_idx), t);
+      rescan();
+    }
+    __syncthreads();
+  };
+
+  int32_t* order = P.order ? P.order + u.unit * B : nullptr;
+  float* margins = P.margins ? P.margins + u.unit * B : nullptr;
+  int t = 0;
+  while (t < nsel) {
+    block_best(my_key, my_idx, sh);
+    const int bi = static_cast<int>(sh.best_idx);
+    if (applied[bi] < t) {            // a stale bound: bring stale bests up to date, search again
+      refresh_stale_bests(t);
+      continue;
+    }
+    // bi is the full greedy's admission at step t
+    const float vstar = v[bi];
+    __syncthreads();                  // every thread has read v[bi] and applied[bi]
+    if (tid == 0) {
+      adm[t] = bi;
+      v[bi] = -INFINITY;
+      if (order) order[t] = bi;
+    }
+    __syncthreads();
+    if (tid == (bi % kAllThreads)) rescan();
+    if (margins) {
+      // the runner-up, brought up to date against admissions 0 .. t-1
+      for (;;) {
+        block_best(my_key, my_idx, sh);
+        const uint32_t si = sh.best_idx;
+        if (si == 0xFFFFFFFFu) {
+          if (tid == 0) margins[t] = INFINITY;
+          break;
+        }
+        if (applied[si] < t) {
+          refresh_stale_bests(t);
+          continue;
+        }
+        if (tid == 0) margins[t] = vstar - v[si];
+        break;
+      }
+    }
+    if (tid == 0) adm_inv[t] = cinv[bi].y;   // inverse norm of the admitted key
+    __syncthreads();
+    ++t;
+    if (!lazy && t < nsel) {
+      // lambda2 > 0: values grow with corr, so every candidate is brought up to date
+      for (int i = tid; i < C; i += kAllThreads)
+        if (v[i] != -INFINITY) refresh(i, t);
+      __syncthreads();
+      rescan();
+    }
+  }
+
+  // 3. admitted positions ascending, then -1 (nsel <= kMaxAllBudget admissions)
+  __syncthreads();
+  int32_t* out = P.indices + u.unit * B;
+  if (tid == 0) {
+    // insertion sort of at most kMaxAllBudget positions (one thread; off the hot path)
+    for (int a = 1; a < nsel; ++a) {
+      const int x = adm[a];
+      int b = a - 1;
+      while (b >= 0 && adm[b] > x) {
+        adm[b + 1] = adm[b];
+        --b;
+      }
+      adm[b + 1] = x;
+    }
+  }
+  __syncthreads();
+  for (int r = tid; r < B; r += kAllThreads) out[r] = r < nsel ? adm[r] : -1;
+  if (order)
+    for (int r = nsel + tid; r < B; r += kAllThreads) order[r] = -1;
+  if (margins)
+    for (int r = nsel + tid; r < B; r += kAllThreads) margins[r] = 0.f;
+}
+
+}  // namespace
+
+cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {
+  constexpr size_t smem = kMaxAllCand * (sizeof(float) + sizeof(uint16_t)) +
+                          kMaxAllBudget * (sizeof(int32_t) + sizeof(float));
+  cudaError_t e = cudaFuncSetAttribute(select_all_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  select_all_kernel<<<static_cast<unsigned>(plan.geo.n_units), kAllThreads, smem, stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace kve

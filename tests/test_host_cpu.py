@@ -168,3 +168,25 @@ def test_plan_ex_flags_without_gpu():
     assert lib.kv_evict_plan_ex(ctypes.byref(cfg), lens, 1, None, 0, ctypes.byref(h),
                                 ctypes.byref(ws)) == K.KVE_OK
     lib.kv_evict_plan_destroy(h)
+
+
+def test_every_candidate_plan_limits_without_gpu():
+    """candidate_factor = 0: pools up to 512 candidates use the pooled selector; longer
+    prefixes the every-candidate selector (Lc <= 32768, B <= 1024, with its own scratch
+    in the workspace); multi-profile selection is refused for such plans."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    small = K.Plan(_spec(candidate_factor=0), [500])
+    big = K.Plan(_spec(candidate_factor=0), [5000])
+    pooled = K.Plan(_spec(candidate_factor=4), [5000])
+    assert big.workspace_bytes > pooled.workspace_bytes
+    assert small.workspace_bytes > 0
+    for spec, lens in [(_spec(candidate_factor=0), [32768 + 32 + 1]),
+                       (_spec(candidate_factor=0, budget=1025), [5000])]:
+        with pytest.raises(K.KvEvictError) as e:
+            K.Plan(spec, lens)
+        assert e.value.status == K.KVE_EINVAL
+    K.Plan(_spec(candidate_factor=0), [32768 + 32])   # Lc = 32768: the largest
+    with pytest.raises(K.KvEvictError) as e:
+        big.select_profiles_workspace(2)
+    assert e.value.status == K.KVE_EINVAL

@@ -288,6 +288,20 @@ def test_near_constant_columns_two_pass(window, L):
     _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
 
 
+@pytest.mark.parametrize("L,B,lams", [(1500, 32, (0.5, -0.5)), (5000, 24, (0.3, 0.6)),
+                                      (2600, 40, (0.0, 0.0)), (700, 8, (-0.3, -3.0))])
+def test_every_candidate_greedy(L, B, lams):
+    """candidate_factor = 0 beyond the 512-slot pool (the unrestricted ablation of
+    Section 3.2): the every-candidate selector -- bounds brought up to date on demand
+    for lambda2 <= 0, every value after each admission for lambda2 > 0 -- against the
+    oracle's full greedy over all Lc candidates, margins included."""
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[L], budget=B, candidate_factor=0,
+                  lambdas=("global",) + lams)
+    batch = synth.make_batch(spec, seed=L + B)
+    plan, bufs, _, lam = _run(spec, batch)
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
 def test_repeatable_bitwise():
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[3000, 700])
     batch = synth.make_batch(spec, seed=11)
