@@ -39,8 +39,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "124d6003395a65bd4e61eec57fcf041e3a6206c79d51b6b7ff4863ee99248673",
-                 "bytes_per_launch": 2178174720 + 74808576}
+SCORE_TRAFFIC = {"source_sha256": "2be5b0f4139bcf8f3bb0ef9b6344e3286be38fead01c6b82573ef65cae19be12",
+                 "bytes_per_launch": 2172432384 + 74367232}
 
 
 def _score_source_sha():
