@@ -822,8 +822,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         int64_t next_unit = -1;   // the next item is a phase-1 item of this unit, not staged
         uint64_t t0 = 0;
         for (;;) {
-          if (__all_sync(0xffffffffu, mbar_try_wait(&ctl.pub_full[slot], par))) break;
-          if (!next_checked && __all_sync(0xffffffffu, mbar_try_wait(&ctl.item_full[nslot], npar))) {
+          // test_wait, not try_wait: the loop also polls the next item's normalisers and
+          // must not be suspended while the epilogue finishes
+          if (__all_sync(0xffffffffu, mbar_test_wait(&ctl.pub_full[slot], par))) break;
+          if (!next_checked && __all_sync(0xffffffffu, mbar_test_wait(&ctl.item_full[nslot], npar))) {
             const int64_t pn = ctl.item_ring[nslot].p;
             const int phn = ctl.item_ring[nslot].phase;
             if (pn < 0 || phn == 0) {
