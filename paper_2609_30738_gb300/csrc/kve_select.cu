@@ -49,8 +49,16 @@ template <int NT>
 struct SelSmall {
   uint32_t warp_tot[NT / 32];
   uint32_t red[2][NT / 32][4];   // per warp: best key, best slot, second key
-  uint32_t prefix, need, cnt, maxkey, teq;
+  uint32_t prefix, need, cnt, maxkey, teq, ncand;
 };
+
+// (key, position) pairs of the threshold bin staged in shared memory, after the
+// finer-digit histogram in the `big` region
+template <int NT>
+__host__ __device__ constexpr uint32_t kCandCap() {
+  return static_cast<uint32_t>((kChunks * NT * sizeof(uint4) - kBins * sizeof(uint32_t)) /
+                               (sizeof(uint32_t) + sizeof(int32_t)));
+}
 
 // Exclusive prefix count of `flag` over the block in thread order; the block
 // total is returned in *total (all threads).
@@ -232,10 +240,16 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   }
   __syncthreads();
 
-  // 2. radix select of the C-th largest key: digits of 12, 12 and 8 bits
-  uint32_t pmask = 0;
-#pragma unroll 1
-  for (int pass = 0; pass < 3; ++pass) {
+  // 2. radix select of the C-th largest key: digits of 12, 12 and 8 bits. The first
+  //    digit's histogram came with the pooling; after it one scan sends every key
+  //    above the threshold bin to the pool and copies the keys of that bin (key,
+  //    position) to shared memory, where the two finer digits and the ties are
+  //    resolved. A bin larger than the copy falls back to scans of the global keys.
+  uint32_t* cand_k = reinterpret_cast<uint32_t*>(big + kBins * sizeof(uint32_t));
+  int32_t* cand_p = reinterpret_cast<int32_t*>(cand_k + kCandCap<NT>());
+  // histogram of the digit at `shift` over the keys matching the prefix, then the
+  // digit where the count from the top first reaches `need`
+  auto digit_pass = [&](int pass, uint32_t pmask, bool staged, uint32_t ncand) {
     const int shift = pass == 0 ? 20 : (pass == 1 ? 8 : 0);
     const int nb = pass == 2 ? 256 : kBins;
     uint32_t* hist = pass == 0 ? hist0 : hist12;
@@ -243,7 +257,13 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       for (int b = tid; b < nb; b += NT) hist[b] = 0;
     __syncthreads();
     const uint32_t prefix = sh.prefix;
-    for (int i0 = 0; pass > 0 && i0 < Lc; i0 += NT * kBatch) {
+    if (pass > 0 && staged) {
+      for (uint32_t e = tid; e < ncand; e += NT) {
+        const uint32_t k = cand_k[e];
+        if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & static_cast<uint32_t>(nb - 1)], 1u);
+      }
+    }
+    for (int i0 = 0; pass > 0 && !staged && i0 < Lc; i0 += NT * kBatch) {
       uint32_t kb[kBatch];
 #pragma unroll
       for (int j = 0; j < kBatch; ++j) {
@@ -258,8 +278,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       }
     }
     __syncthreads();
-    // thread t owns bins [t*per, (t+1)*per); find the digit where the count from
-    // the top first reaches `need`
+    // thread t owns bins [t*per, (t+1)*per)
     const int per = nb / NT > 0 ? nb / NT : 1;
     const int b0 = tid * per;
     uint32_t mine = 0;
@@ -279,32 +298,86 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
         acc += c;
       }
     }
-    pmask |= static_cast<uint32_t>(nb - 1) << shift;
     __syncthreads();
+  };
+  digit_pass(0, 0u, false, 0u);
+  // the scan: keys above the first digit's bin go to the pool, that bin to `cand`
+  if (tid == 0) {
+    sh.cnt = 0;
+    sh.ncand = 0;
   }
+  __syncthreads();
+  {
+    const uint32_t bin = sh.prefix >> 20;
+    for (int i0 = 0; i0 < Lc; i0 += NT * kBatch) {
+      uint32_t kb[kBatch];
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        kb[j] = i < Lc ? __ldcg(&keys[i]) : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        if (i < Lc) {
+          const uint32_t d = kb[j] >> 20;
+          if (d > bin) {
+            cpos[atomicAdd(&sh.cnt, 1u)] = i;
+          } else if (d == bin) {
+            const uint32_t e = atomicAdd(&sh.ncand, 1u);
+            if (e < kCandCap<NT>()) {
+              cand_k[e] = kb[j];
+              cand_p[e] = i;
+            }
+          }
+        }
+      }
+    }
+  }
+  __syncthreads();
+  const uint32_t ncand = sh.ncand;
+  const bool staged = ncand <= kCandCap<NT>();
+  digit_pass(1, 0xFFFu << 20, staged, ncand);
+  digit_pass(2, 0xFFFFFFu << 8, staged, ncand);
   const uint32_t T = sh.prefix;
   const uint32_t needT = sh.need;   // keys equal to T to take, lowest positions first
 
   // 3. every key above the threshold, and the positions of the keys equal to it
-  if (tid == 0) sh.teq = 0;
+  //    (the tie list overlays the dead finer-digit histogram)
+  int32_t* ties = reinterpret_cast<int32_t*>(big);   // [kTieCap]
+  if (tid == 0) {
+    sh.teq = 0;
+    if (!staged) sh.cnt = 0;   // the global scans below collect the whole pool again
+  }
   __syncthreads();
-  int32_t* ties = reinterpret_cast<int32_t*>(big);   // [kTieCap], the histogram is dead
-  for (int i0 = 0; i0 < Lc; i0 += NT * kBatch) {
-    uint32_t kb[kBatch];
-#pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int i = i0 + j * NT + tid;
-      kb[j] = i < Lc ? __ldcg(&keys[i]) : 0u;
+  if (staged) {
+    for (uint32_t e = tid; e < ncand; e += NT) {
+      const uint32_t k = cand_k[e];
+      if (k > T) {
+        cpos[atomicAdd(&sh.cnt, 1u)] = cand_p[e];
+      } else if (k == T) {
+        const uint32_t q = atomicAdd(&sh.teq, 1u);
+        if (q < kTieCap) ties[q] = cand_p[e];
+      }
     }
+  } else {
+    for (int i0 = 0; i0 < Lc; i0 += NT * kBatch) {
+      uint32_t kb[kBatch];
 #pragma unroll
-    for (int j = 0; j < kBatch; ++j) {
-      const int i = i0 + j * NT + tid;
-      if (i < Lc) {
-        if (kb[j] > T) {
-          cpos[atomicAdd(&sh.cnt, 1u)] = i;
-        } else if (kb[j] == T) {
-          const uint32_t e = atomicAdd(&sh.teq, 1u);
-          if (e < kTieCap) ties[e] = i;
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        kb[j] = i < Lc ? __ldcg(&keys[i]) : 0u;
+      }
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int i = i0 + j * NT + tid;
+        if (i < Lc) {
+          if (kb[j] > T) {
+            cpos[atomicAdd(&sh.cnt, 1u)] = i;
+          } else if (kb[j] == T) {
+            const uint32_t e = atomicAdd(&sh.teq, 1u);
+            if (e < kTieCap) ties[e] = i;
+          }
         }
       }
     }

@@ -275,12 +275,16 @@ def test_edge_shapes(L, B, pk, cf):
     _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
 
 
-@pytest.mark.parametrize("window,L", [(32, 2048), (8, 1500)])
+@pytest.mark.parametrize("window,L", [(32, 2048), (8, 1500), (32, 8192)])
 def test_near_constant_columns_two_pass(window, L):
     """Zero window queries: every row spreads its mass evenly over its causal prefix,
     so each column's A values differ only through the rows' prefix lengths
     (sigma/mu ~ W / L). The one-pass sums cannot be trusted there and every warp
-    takes the two-pass form; mu and sigma still meet the tolerances."""
+    takes the two-pass form; mu and sigma still meet the tolerances. Every prefix
+    key then has the same base score: at L = 8192 the threshold bin of the
+    selector's radix select (8160 keys) exceeds its shared-memory copy and the cut
+    falls among more equal keys than the tie list holds, so the global-scan paths
+    run."""
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], window=window, budget=16, seq_lens=[L])
     batch = synth.make_batch(spec, seed=31)
     batch["q_win"] = torch.zeros_like(batch["q_win"])
