@@ -303,7 +303,7 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
                            const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
                            float* margins, void* ws, void* stream) {
   if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws) return KVE_EINVAL;
-  if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(mu, 16) || !aligned(sigma, 16) || !aligned(ws, 256)) return KVE_EINVAL;
   kve::SelectParams p;
   const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
   if (s != KVE_OK) return s;
@@ -329,7 +329,7 @@ kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles, co
   if (!plan || n_profiles < 1 || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || !ws ||
       plan->select_all)
     return KVE_EINVAL;
-  if (!aligned(k, 16) || !aligned(ws, 256)) return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(mu, 16) || !aligned(sigma, 16) || !aligned(ws, 256)) return KVE_EINVAL;
   const int32_t nl = plan->geo.num_layers;
   for (int64_t i = 0; i < static_cast<int64_t>(n_profiles) * nl; ++i)
     if (!std::isfinite(lambda1[i]) || !std::isfinite(lambda2[i])) return KVE_EINVAL;

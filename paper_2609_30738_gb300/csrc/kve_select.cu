@@ -40,6 +40,13 @@ __device__ __forceinline__ uint32_t ord_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
+// max of three floats in one instruction
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 __device__ __forceinline__ float unord_key(uint32_t k) {
   const uint32_t u = (k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k;
   return __uint_as_float(u);
@@ -151,10 +158,83 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
 
   for (int b = tid; b < kBins; b += NT) hist0[b] = 0;
   __syncthreads();
-  // 1. pooled base score as ordered keys (and the histogram of their top 12 bits);
-  //    a tile holds kPoolRuns runs of kPoolRun
-  //    consecutive outputs per thread (run q of thread t starts at (q*NT + t)*kPoolRun)
-  {
+  // 1. pooled base score as ordered keys (and the histogram of their top 12 bits)
+  if (h == 3) {
+    // kernel 7 (the default): groups of 4 consecutive outputs that are 16-byte
+    // aligned in mu, sigma and keys, each from three 16-byte loads per array (inputs
+    // i-4 .. i+7); groups at the ends of the range take their inputs one by one
+    const int lead = static_cast<int>(u.mu_off & 3);   // unit elements before its first aligned group
+    const int ngroups = (lead + Lc + 3) / 4;
+    for (int q = tid; q < ngroups; q += NT) {
+      const int i = 4 * q - lead;                      // first output of the group (may be < 0)
+      float xm[12], xs[12];                            // positions i-4 .. i+7
+      if (i >= 4 && i + 8 <= Lc) {
+        const float4* m4 = reinterpret_cast<const float4*>(mu + i - 4);
+        const float4* s4 = reinterpret_cast<const float4*>(sg + i - 4);
+#pragma unroll
+        for (int c = 0; c < 3; ++c) {
+          const float4 am = __ldg(m4 + c), as = __ldg(s4 + c);
+          xm[4 * c] = am.x;
+          xm[4 * c + 1] = am.y;
+          xm[4 * c + 2] = am.z;
+          xm[4 * c + 3] = am.w;
+          xs[4 * c] = as.x;
+          xs[4 * c + 1] = as.y;
+          xs[4 * c + 2] = as.z;
+          xs[4 * c + 3] = as.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 12; ++j) {
+          const int pj = i - 4 + j;
+          const bool in = pj >= 0 && pj < Lc;          // the window is clipped to [0, Lc)
+          xm[j] = in ? __ldg(mu + pj) : -INFINITY;
+          xs[j] = in ? __ldg(sg + pj) : -INFINITY;
+        }
+      }
+      // output r (position i + r) pools positions i+r-3 .. i+r+3 = x[r+1 .. r+7]
+      const float cm = fmaxf(max3(xm[4], xm[5], xm[6]), xm[7]);
+      const float cs = fmaxf(max3(xs[4], xs[5], xs[6]), xs[7]);
+      float om[4], os[4];
+      om[0] = fmaxf(max3(cm, xm[1], xm[2]), xm[3]);
+      om[1] = fmaxf(max3(cm, xm[2], xm[3]), xm[8]);
+      om[2] = fmaxf(max3(cm, xm[3], xm[8]), xm[9]);
+      om[3] = fmaxf(max3(cm, xm[8], xm[9]), xm[10]);
+      os[0] = fmaxf(max3(cs, xs[1], xs[2]), xs[3]);
+      os[1] = fmaxf(max3(cs, xs[2], xs[3]), xs[8]);
+      os[2] = fmaxf(max3(cs, xs[3], xs[8]), xs[9]);
+      os[3] = fmaxf(max3(cs, xs[8], xs[9]), xs[10]);
+      uint32_t kk[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) kk[r] = ord_key(fmaf(lambda1, os[r], om[r]));
+      if (i >= 0 && i + 4 <= Lc) {
+        *reinterpret_cast<uint4*>(keys + i) = make_uint4(kk[0], kk[1], kk[2], kk[3]);
+        // consecutive outputs often share the top digit: one atomic per run
+        uint32_t bin = kk[0] >> 20, cnt = 1;
+#pragma unroll
+        for (int r = 1; r < 4; ++r) {
+          const uint32_t br = kk[r] >> 20;
+          if (br == bin) {
+            ++cnt;
+          } else {
+            atomicAdd(&hist0[bin], cnt);
+            bin = br;
+            cnt = 1;
+          }
+        }
+        atomicAdd(&hist0[bin], cnt);
+      } else {
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          if (i + r >= 0 && i + r < Lc) {
+            keys[i + r] = kk[r];
+            atomicAdd(&hist0[kk[r] >> 20], 1u);
+          }
+      }
+    }
+  } else {
+    // any other kernel: a tile holds kPoolRuns runs of kPoolRun consecutive outputs
+    // per thread (run q of thread t starts at (q*NT + t)*kPoolRun)
     constexpr int kTile = NT * kPoolRun * kPoolRuns;
     const int tile_in = kTile + 2 * h;
     float* tsg = tmu + tile_in;
@@ -667,7 +747,9 @@ extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float*
   const Geometry& g = plan->geo;
   const size_t words = static_cast<size_t>(g.num_layers) * g.uheads * static_cast<size_t>(g.total_tokens);
   if (words > kNoAllocScratchWords) return KVE_EINVAL;   // beyond the fixed scratch
-  if ((reinterpret_cast<uintptr_t>(k) & 15u) != 0) return KVE_EINVAL;
+  if (((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(mu) |
+        reinterpret_cast<uintptr_t>(sigma)) & 15u) != 0)
+    return KVE_EINVAL;   // the header asks every pointer to be 16-byte aligned
   uint32_t* scratch = scratch_on_current_device();
   if (!scratch) return KVE_ECUDA;
   SelectParams p;

@@ -72,6 +72,15 @@ def test_null_arguments_rejected_without_gpu():
     assert lib.kv_evict_gather(None, None, None, None, None, None, None) == K.KVE_EINVAL
     assert lib.kv_evict_plan_set_debug(p._h, 0, 0) == K.KVE_EINVAL
     assert lib.kv_evict_strerror(K.KVE_ETIMEOUT) == b"device-side wait timed out"
+    # mu / sigma must be 16-byte aligned (the selector reads them 16 bytes at a time);
+    # the check fails before any launch, so fake device addresses suffice
+    lam = np.zeros(2, np.float32)
+    good, odd = ctypes.c_void_p(1 << 20), ctypes.c_void_p((1 << 20) + 4)
+    for mu, sg in [(odd, good), (good, odd)]:
+        assert lib.kv_evict_select(p._h, mu, sg, good, lam.ctypes.data, lam.ctypes.data, good, None, None,
+                                   good, None) == K.KVE_EINVAL
+        assert lib.kv_evict_select_noalloc(p._h, mu, sg, good, lam.ctypes.data, lam.ctypes.data, good, None,
+                                           None, None) == K.KVE_EINVAL
 
 
 @pytest.mark.parametrize("kind,c", [("global", [0.3]), ("segments", [-0.8, 0.6, -0.8]),
