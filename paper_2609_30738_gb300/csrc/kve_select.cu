@@ -165,9 +165,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     // i-4 .. i+7); groups at the ends of the range take their inputs one by one
     const int lead = static_cast<int>(u.mu_off & 3);   // unit elements before its first aligned group
     const int ngroups = (lead + Lc + 3) / 4;
-    for (int q = tid; q < ngroups; q += NT) {
-      const int i = 4 * q - lead;                      // first output of the group (may be < 0)
-      float xm[12], xs[12];                            // positions i-4 .. i+7
+    // inputs of group q: positions 4q-lead-4 .. 4q-lead+7
+    auto load_group = [&](int q, float (&xm)[12], float (&xs)[12]) {
+      const int i = 4 * q - lead;
       if (i >= 4 && i + 8 <= Lc) {
         const float4* m4 = reinterpret_cast<const float4*>(mu + i - 4);
         const float4* s4 = reinterpret_cast<const float4*>(sg + i - 4);
@@ -192,7 +192,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
           xs[j] = in ? __ldg(sg + pj) : -INFINITY;
         }
       }
-      // output r (position i + r) pools positions i+r-3 .. i+r+3 = x[r+1 .. r+7]
+    };
+    // output r (position i + r) pools positions i+r-3 .. i+r+3 = x[r+1 .. r+7]
+    auto emit_group = [&](int q, const float (&xm)[12], const float (&xs)[12]) {
+      const int i = 4 * q - lead;
       const float cm = fmaxf(max3(xm[4], xm[5], xm[6]), xm[7]);
       const float cs = fmaxf(max3(xs[4], xs[5], xs[6]), xs[7]);
       float om[4], os[4];
@@ -231,6 +234,15 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
             atomicAdd(&hist0[kk[r] >> 20], 1u);
           }
       }
+    };
+    // two groups per pass: their loads are in flight together
+    for (int q = tid; q < ngroups; q += 2 * NT) {
+      float xm0[12], xs0[12], xm1[12], xs1[12];
+      const bool two = q + NT < ngroups;
+      load_group(q, xm0, xs0);
+      if (two) load_group(q + NT, xm1, xs1);
+      emit_group(q, xm0, xs0);
+      if (two) emit_group(q + NT, xm1, xs1);
     }
   } else {
     // any other kernel: a tile holds kPoolRuns runs of kPoolRun consecutive outputs
