@@ -231,23 +231,17 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
     }
   }
 
-  // 3. admitted positions ascending, then -1 (nsel <= kMaxAllBudget admissions)
+  // 3. admitted positions ascending, then -1: entry a of the admission order goes to
+  //    its rank among the admitted positions (all distinct); nsel <= kMaxAllBudget
   __syncthreads();
   int32_t* out = P.indices + u.unit * B;
-  if (tid == 0) {
-    // insertion sort of at most kMaxAllBudget positions (one thread; off the hot path)
-    for (int a = 1; a < nsel; ++a) {
-      const int x = adm[a];
-      int b = a - 1;
-      while (b >= 0 && adm[b] > x) {
-        adm[b + 1] = adm[b];
-        --b;
-      }
-      adm[b + 1] = x;
-    }
+  for (int a = tid; a < nsel; a += kAllThreads) {
+    const int pos = adm[a];
+    int rank = 0;
+    for (int c = 0; c < nsel; ++c) rank += (adm[c] < pos);
+    out[rank] = pos;
   }
-  __syncthreads();
-  for (int r = tid; r < B; r += kAllThreads) out[r] = r < nsel ? adm[r] : -1;
+  for (int r = nsel + tid; r < B; r += kAllThreads) out[r] = -1;
   if (order)
     for (int r = nsel + tid; r < B; r += kAllThreads) order[r] = -1;
   if (margins)

@@ -173,6 +173,57 @@ def test_per_query_head_selection_every_unit():
                                 idx_all[ui], L, W, B)
 
 
+def test_per_query_head_combinations():
+    """A per-query-head plan with per-layer budgets: multi-profile selection and the
+    workspace-free selection give kv_evict_select's outputs bit for bit, and the
+    selection replays through the oracle at each layer's budget."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    lb = K.budget_pyramid(16, 3, 0.5)            # [24, 16, 8]
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=3, budget=int(lb[0]), seq_lens=[800, 1100])
+    batch = synth.make_batch(spec, seed=47)
+    seq = batch["seq_lens"]
+    plan = K.Plan(spec, seq, layer_budgets=lb, per_query_head=True)
+    bufs = K.Buffers(plan)
+    lam = lambda_arrays(spec, K.profile)
+    q, k, v = (batch[x].to(DEV) for x in ("q_win", "k", "v"))
+    K.run_step(plan, bufs, q, k, v, lam[0], lam[1])
+    assert plan.status(bufs.ws) == K.KVE_OK
+    U, B = plan.n_units, spec["budget"]
+    l1 = np.stack([lam[0], lam[0] * 0.5]).astype(np.float32)
+    l2 = np.stack([lam[1], lam[1] * 2.0]).astype(np.float32)
+    idx = torch.empty((2, U, B), dtype=torch.int32, device=DEV)
+    ws = torch.empty(plan.select_profiles_workspace(2), dtype=torch.uint8, device=DEV)
+    plan.select_profiles(bufs.mu, bufs.sigma, k, l1, l2, idx, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(idx[0], bufs.indices)
+    idx_na = torch.empty_like(bufs.indices)
+    plan.select_noalloc(bufs.mu, bufs.sigma, k, l1[1], l2[1], idx_na)
+    torch.cuda.synchronize()
+    assert torch.equal(idx[1], idx_na)
+    # layer 2 of request 1, query head 13, against the oracle
+    W, Hq, G, N_L = spec["window"], spec["num_q_heads"], 4, 3
+    r, layer, hq = 1, 2, 13
+    L, off = seq[r], sum(seq[:r])
+    qb = PT.to_bits(batch["q_win"][layer, r, hq]).reshape(W, -1)
+    kb = PT.to_bits(batch["k"][layer, hq // G, off:off + L])
+    kf = O.bf16_bits_to_f64(kb)
+    mu_ref, sg_ref = O.score_unit(O.bf16_bits_to_f64(qb), kf, L, W, 1)
+    ui = (r * N_L + layer) * Hq + hq
+    PT.check_selection(bufs.order[ui].cpu().numpy(), bufs.indices[ui].cpu().numpy(), mu_ref, sg_ref, kf, L, W,
+                       int(lb[layer]), float(lam[0][layer]), float(lam[1][layer]), spec["pool_kernel"],
+                       spec["candidate_factor"], spec["norm_eps"], margins_gpu=bufs.margins[ui].cpu().numpy())
+
+
+def test_every_candidate_with_layer_budgets():
+    """The every-candidate selector at each layer's own budget (B_l < B)."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=24, candidate_factor=0,
+                  seq_lens=[1300])
+    batch = synth.make_batch(spec, seed=53)
+    plan, bufs, _, lam = _run(spec, batch, layer_budgets=[24, 9])
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+
+
 def test_per_query_head_equals_default_without_grouping():
     """With one query head per KV head (G = 1) both readings define the same units:
     the per-query-head plan gives the default plan's outputs bit for bit."""
