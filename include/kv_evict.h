@@ -204,7 +204,9 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k,
                            uint16_t* k_out, uint16_t* v_out, void* stream);
 
 /* Synchronise the stream, read the device error word of ws and clear it.
- * Returns KVE_OK, KVE_ETIMEOUT or KVE_ECUDA. */
+ * Returns KVE_OK, KVE_ETIMEOUT (a bounded wait ran out) or KVE_ECUDA (a CUDA call
+ * failed, or a device-side consistency check of kv_evict_select failed: a pool
+ * position outside the unit, whose key row is then not read). */
 kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream);
 
 /* Depth profile of Eq. 6 on the host: kind 0 Global (lambda = sinh(c[0]) on every

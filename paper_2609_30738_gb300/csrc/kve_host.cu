@@ -308,6 +308,7 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
   const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
   if (s != KVE_OK) return s;
   p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.keys);
+  p.err = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.hdr);
   if (plan->select_all) {
     p.corr = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + plan->ws.corr);
     return kve::launch_select_all(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK
@@ -383,7 +384,7 @@ kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream) {
   if (cudaMemcpy(&err, ws, sizeof(err), cudaMemcpyDeviceToHost) != cudaSuccess) return KVE_ECUDA;
   if (err != 0) {
     if (cudaMemset(ws, 0, sizeof(err)) != cudaSuccess) return KVE_ECUDA;
-    return KVE_ETIMEOUT;
+    return (err & kve::kErrCheck) ? KVE_ECUDA : KVE_ETIMEOUT;
   }
   return KVE_OK;
 }

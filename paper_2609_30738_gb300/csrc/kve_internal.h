@@ -20,6 +20,9 @@ constexpr int kMaxLayers = 256;    // layers per call (lambda arrays ride in ker
 constexpr int kMaxPoolCand = 512;  // candidate pool of the pooled selector (shared memory)
 constexpr int kMaxAllCand = 32768; // candidates of the every-candidate selector (Lc)
 constexpr int kMaxAllBudget = 1024;// admissions of the every-candidate selector
+// Bits of the workspace error word (kv_evict_status).
+constexpr uint32_t kErrWait = 1u;    // a bounded wait ran out
+constexpr uint32_t kErrCheck = 2u;   // a device-side consistency check failed
 
 // Request table and derived counts, identical on host and device.
 struct Geometry {
@@ -131,6 +134,7 @@ struct SelectParams {
   int32_t* order;
   float* margins;
   uint32_t* keys;            // workspace scratch
+  uint32_t* err;             // workspace error word (or null): bit 2 = a pool position out of range
   float* corr;               // workspace scratch of the every-candidate selector (or null):
                              // float2 (corr, 1/|k|) per prefix token of every unit
   float lambda1[kMaxLayers];

@@ -144,7 +144,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   uint32_t* keys = P.keys + keys_off + u.mu_off;
   const int h = P.pool_kernel / 2;
 
-  // shared memory: [ big | spos | cpos | st | inv ]; `big` holds in turn the pooling
+  // shared memory: [ big | spos | cpos | inv | hist0 ]; `big` holds in turn the pooling
   // tiles, the radix histogram and the staged candidate keys
   uint8_t* big = dyn;
   uint4* krow = reinterpret_cast<uint4*>(big);                                  // [NT][kChunks]
@@ -152,8 +152,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   float* tmu = reinterpret_cast<float*>(big);                                   // pooling tiles
   int32_t* spos = reinterpret_cast<int32_t*>(big + kChunks * NT * sizeof(uint4));
   int32_t* cpos = spos + NT;
-  float* st = reinterpret_cast<float*>(cpos + NT);
-  float* inv = st + NT;
+  float* inv = reinterpret_cast<float*>(cpos + NT);
   uint32_t* hist0 = reinterpret_cast<uint32_t*>(inv + NT);                      // [kBins] first pass
 
   for (int b = tid; b < kBins; b += NT) hist0[b] = 0;
@@ -519,8 +518,13 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       const int r = (q * (NT / 32) + warp) * 2 + (lane >> 4);
       xr[q] = make_uint4(0, 0, 0, 0);
       if (r < C) {
-        const uint4* src = reinterpret_cast<const uint4*>(P.k + (u.k_row0 + spos[r]) * kHeadDim);
-        xr[q] = __ldg(src + (lane & 15));
+        const int pos = spos[r];
+        if (pos >= 0 && pos < Lc) {
+          const uint4* src = reinterpret_cast<const uint4*>(P.k + (u.k_row0 + pos) * kHeadDim);
+          xr[q] = __ldg(src + (lane & 15));
+        } else if (P.err) {
+          atomicOr(P.err, kErrCheck);   // never read outside the unit's keys
+        }
       }
     }
 #pragma unroll
@@ -662,8 +666,8 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
 
 template <int NT>
 constexpr size_t select_smem() {
-  // candidate keys (also reused for the pooling tiles and the histogram) + 4 arrays
-  return kChunks * NT * sizeof(uint4) + 4 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
+  // candidate keys (also reused for the pooling tiles and the histogram) + 3 arrays
+  return kChunks * NT * sizeof(uint4) + 3 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
 }
 static_assert(kChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histogram fits");
 static_assert(kChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),

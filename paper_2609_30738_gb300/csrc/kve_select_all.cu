@@ -40,7 +40,6 @@ struct AllSmall {
   uint32_t widx[kAllWarps];
   float wmax[kAllWarps];
   uint32_t best_key, best_idx;
-  int32_t refreshed;
 };
 
 // Block argmax of the owners' bests: the largest key, ties to the lowest index.
