@@ -337,13 +337,24 @@ def run_ours(args):
         o_k = torch.empty_like(bufs.k_out, device="cpu").pin_memory()
         o_v = torch.empty_like(bufs.v_out, device="cpu").pin_memory()
         dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+        # V is needed only by the gather: its copy runs on a second stream, beside the
+        # copy of Q and K and the score and select kernels
+        side = torch.cuda.Stream(device=dev)
+        v_ready = torch.cuda.Event()
 
         def e2e_step():
+            side.wait_stream(stream)           # the previous step's gather has read dv
+            with torch.cuda.stream(side):
+                dv.copy_(hv, non_blocking=True)
+                v_ready.record(side)
             with torch.cuda.stream(stream):
                 dq.copy_(hq, non_blocking=True)
                 dk.copy_(hk, non_blocking=True)
-                dv.copy_(hv, non_blocking=True)
-            K.run_step(plan, bufs, dq, dk, dv, lam1, lam2, stream=stream)
+            plan.score(dq, dk, bufs.mu, bufs.sigma, bufs.ws, stream)
+            plan.select(bufs.mu, bufs.sigma, dk, lam1, lam2, bufs.indices, bufs.ws, bufs.order,
+                        bufs.margins, stream)
+            stream.wait_event(v_ready)
+            plan.gather(dk, dv, bufs.indices, bufs.k_out, bufs.v_out, stream)
             with torch.cuda.stream(stream):
                 o_idx.copy_(bufs.indices, non_blocking=True)
                 o_k.copy_(bufs.k_out, non_blocking=True)
