@@ -393,13 +393,13 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- sync warp
 
-// One round of loads of a unit's tagged normalisers (4 rows per lane); rows past n
-// read as ready.
+// One round of loads of a unit's tagged normalisers (4 rows per lane; relaxed GPU-scope
+// loads, so that every poll reads memory again); rows past n read as ready.
 __device__ __forceinline__ void load_beta(const ScoreParams& P, int64_t unit, unsigned long long w[4]) {
   const int r0 = 4 * (threadIdx.x & 31);
 #pragma unroll
   for (int k = 0; k < 4; ++k)
-    w[k] = (r0 + k < P.g.n_rows) ? __ldcg(&P.beta[unit * kMaxRows + r0 + k]) : (1ull << 32);
+    w[k] = (r0 + k < P.g.n_rows) ? ld_relaxed_gpu_u64(&P.beta[unit * kMaxRows + r0 + k]) : (1ull << 32);
 }
 
 // If every row of w is tagged ready, stage -beta for the epilogue and return true.
