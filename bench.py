@@ -39,8 +39,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "2be5b0f4139bcf8f3bb0ef9b6344e3286be38fead01c6b82573ef65cae19be12",
-                 "bytes_per_launch": 2172432384 + 74367232}
+SCORE_TRAFFIC = {"source_sha256": "a7780fdb74b52d1e107310669b775c1e30f31d00900ec431d979bcd57b71e4bb",
+                 "bytes_per_launch": 2172929024 + 74867200}
 
 
 def _score_source_sha():
