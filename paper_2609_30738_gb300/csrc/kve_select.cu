@@ -586,18 +586,17 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       sh.red[t & 1][warp][2] = wsec;
     }
     __syncthreads();
-    uint32_t best = 0, bslot = 0xFFFFFFFFu, sec = 0;
-#pragma unroll
-    for (int w = 0; w < NT / 32; ++w) {
-      const uint32_t k = sh.red[t & 1][w][0], sl = sh.red[t & 1][w][1], k2 = sh.red[t & 1][w][2];
-      if (k > best || (k == best && sl < bslot)) {
-        sec = max(sec, best);
-        best = k;
-        bslot = sl;
-      } else {
-        sec = max(sec, k);
-      }
-      sec = max(sec, k2);
+    // every warp reduces the NT/32 warp results itself (lane w holds warp w's)
+    const bool hold = lane < NT / 32;
+    const uint32_t k_l = hold ? sh.red[t & 1][lane][0] : 0u;
+    const uint32_t sl_l = hold ? sh.red[t & 1][lane][1] : 0xFFFFFFFFu;
+    const uint32_t best = __reduce_max_sync(0xffffffffu, k_l);
+    const uint32_t bslot = __reduce_min_sync(0xffffffffu, k_l == best ? sl_l : 0xFFFFFFFFu);
+    uint32_t sec = 0;
+    if (margins) {
+      const uint32_t k2_l = hold ? sh.red[t & 1][lane][2] : 0u;
+      // runner-up: the other warps' best and the winning warp's second
+      sec = __reduce_max_sync(0xffffffffu, (k_l == best && sl_l == bslot) ? k2_l : max(k_l, k2_l));
     }
     const int js = static_cast<int>(bslot);
     if (tid == 0) {
