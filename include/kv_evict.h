@@ -198,7 +198,14 @@ kve_status kv_evict_select_noalloc(const kve_plan* plan, const float* mu,
                                    float* margins, void* stream);
 
 /* Step 4: compact cache (Section 1: each layer keeps B entries after prefill;
- * the window tokens are kept as well). Copies key/value rows bit-exactly. */
+ * the window tokens are kept as well). Copies key/value rows bit-exactly.
+ * Exception to the device-memory convention: k and v may also be page-locked
+ * host memory of the CUDA runtime (cudaHostAlloc, cudaMallocHost, or host memory
+ * registered with cudaHostRegister). Under unified addressing the kernel reads
+ * such memory in place, and only the kept rows (min(B_l, Lc_r) + W per unit)
+ * cross the host link. k_out and v_out stay in device memory. Returns KVE_EINVAL
+ * for host memory the runtime does not know (pageable memory) or a pointer the
+ * runtime cannot classify. */
 kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k,
                            const uint16_t* v, const int32_t* indices,
                            uint16_t* k_out, uint16_t* v_out, void* stream);

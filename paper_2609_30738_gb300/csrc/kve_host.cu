@@ -363,6 +363,16 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16
                            uint16_t* k_out, uint16_t* v_out, void* stream) {
   if (!plan || !k || !v || !indices || !k_out || !v_out) return KVE_EINVAL;
   if (!aligned(k, 16) || !aligned(v, 16) || !aligned(k_out, 16) || !aligned(v_out, 16)) return KVE_EINVAL;
+  // k and v may be pinned host memory (read in place under unified addressing);
+  // host memory the CUDA runtime does not know is refused
+  for (const void* src : {static_cast<const void*>(k), static_cast<const void*>(v)}) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, src) != cudaSuccess) {
+      cudaGetLastError();
+      return KVE_EINVAL;
+    }
+    if (at.type == cudaMemoryTypeUnregistered) return KVE_EINVAL;
+  }
   kve::GatherParams p;
   std::memset(&p, 0, sizeof(p));
   p.g = plan->geo;

@@ -222,6 +222,13 @@ class Plan:
                "kv_evict_select_profiles")
 
     def gather(self, k, v, indices, k_out, v_out, stream=None):
+        """kv_evict_gather. k and v may be pinned CPU tensors (read in place by the
+        kernel; only the kept rows cross the host link); pageable CPU tensors are
+        refused."""
+        for name, t in (("k", k), ("v", v)):
+            dev = getattr(t, "device", None)
+            if dev is not None and getattr(dev, "type", None) == "cpu" and not t.is_pinned():
+                raise ValueError(f"gather: {name} is a pageable CPU tensor; pin it or move it to the GPU")
         _check(_lib().kv_evict_gather(self._h, _ptr(k), _ptr(v), _ptr(indices), _ptr(k_out),
                                       _ptr(v_out), _stream_ptr(stream)), "kv_evict_gather")
 

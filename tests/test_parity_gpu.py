@@ -368,6 +368,38 @@ def test_repeatable_bitwise():
     assert torch.equal(idx1, bufs.indices)
 
 
+def test_gather_reads_pinned_host_kv_in_place():
+    """k and v in pinned host memory: the gather reads the kept rows in place and
+    writes the same compact cache, bit for bit, as from the device copies; pageable
+    host memory is refused by the binding and by the C ABI before any launch."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=16,
+                  seq_lens=[300, 1500, 513])
+    batch = synth.make_batch(spec, seed=13)
+    plan, bufs, (q, k, v), lam = _run(spec, batch)
+    ko_dev, vo_dev = bufs.k_out.clone(), bufs.v_out.clone()
+    hk, hv = batch["k"].contiguous().pin_memory(), batch["v"].contiguous().pin_memory()
+    bufs.k_out.fill_(1)
+    bufs.v_out.fill_(1)
+    plan.gather(hk, hv, bufs.indices, bufs.k_out, bufs.v_out)
+    assert plan.status(bufs.ws) == K.KVE_OK
+    assert torch.equal(ko_dev, bufs.k_out) and torch.equal(vo_dev, bufs.v_out)
+    bufs.v_out.fill_(1)
+    plan.gather(k, hv, bufs.indices, bufs.k_out, bufs.v_out)   # k on the device, v on the host
+    assert plan.status(bufs.ws) == K.KVE_OK
+    assert torch.equal(vo_dev, bufs.v_out)
+    pv = batch["v"].contiguous()
+    assert not pv.is_pinned()
+    with pytest.raises(ValueError):
+        plan.gather(k, pv, bufs.indices, bufs.k_out, bufs.v_out)
+    bufs.v_out.fill_(1)
+    st = K.library().kv_evict_gather(plan._h, k.data_ptr(), pv.data_ptr(), bufs.indices.data_ptr(),
+                                     bufs.k_out.data_ptr(), bufs.v_out.data_ptr(), None)
+    assert st == K.KVE_EINVAL
+    torch.cuda.synchronize()
+    assert bool((bufs.v_out == 1).all())   # refused before any launch: nothing written
+
+
 def test_bounded_wait_reports_timeout_and_gpu_stays_usable():
     """A unit whose row statistics are never published (host-set test hook): the
     column pass waits out a 5 ms limit, reports KVE_ETIMEOUT, and the next call
