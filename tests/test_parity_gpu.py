@@ -455,3 +455,37 @@ def test_full_size_sampled_units(name):
                     (len(seq) - 1, 21, 2)})
     worst, swaps = _check_units(spec, batch, plan, bufs, lam, units)
     print(f"{name}: max mu rel err {worst:.2e}, near-tie swaps {swaps}")
+
+
+def test_layer_chunks_with_host_values_full_size():
+    """The end-to-end launch configuration at full size: one plan per chunk of 4
+    layers, working on views into the full arrays, with V read in place from pinned
+    host memory by the gather; sampled units (chunk edges included) against the
+    oracle."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = WORKLOADS["mistral-32layer-L32768-B64"]
+    batch = synth.make_batch(spec, seed=2609, device=DEV)
+    N_L, chunks = spec["num_layers"], 8
+    Lc = N_L // chunks
+    plan = K.Plan(spec, batch["seq_lens"])
+    bufs = K.Buffers(plan)
+    cplan = K.Plan(dict(spec, num_layers=Lc), batch["seq_lens"])
+    cws = torch.empty(cplan.workspace_bytes, dtype=torch.uint8, device=DEV)
+    lam = lambda_arrays(spec, K.profile)
+    q, k = batch["q_win"], batch["k"]
+    hv = batch["v"].cpu().pin_memory()
+    mu_c, sg_c = bufs.mu.view(chunks, -1), bufs.sigma.view(chunks, -1)
+    idx_c, ord_c = bufs.indices.view(chunks, -1, spec["budget"]), bufs.order.view(chunks, -1, spec["budget"])
+    mar_c = bufs.margins.view(chunks, -1, spec["budget"])
+    ko_c = bufs.k_out.view(chunks, -1, *bufs.k_out.shape[1:])
+    vo_c = bufs.v_out.view(chunks, -1, *bufs.v_out.shape[1:])
+    for c in range(chunks):
+        ls = slice(c * Lc, (c + 1) * Lc)
+        cplan.score(q[ls], k[ls], mu_c[c], sg_c[c], cws)
+        cplan.select(mu_c[c], sg_c[c], k[ls], lam[0][ls], lam[1][ls], idx_c[c], cws, ord_c[c], mar_c[c])
+        cplan.gather(k[ls], hv[ls], idx_c[c], ko_c[c], vo_c[c])
+    assert cplan.status(cws) == K.KVE_OK
+    units = [(0, 0, 0), (0, 3, 7), (0, 4, 0), (0, 17, 3), (0, 28, 5), (0, 31, 7)]
+    worst, swaps = _check_units(spec, batch, plan, bufs, lam, units)
+    print(f"layer chunks: max mu rel err {worst:.2e}, near-tie swaps {swaps}")
+
