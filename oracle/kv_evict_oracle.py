@@ -24,7 +24,7 @@ float64 from the bf16-decoded inputs, in the paper's order:
   depth_profile      Eq. 6: a(l) = c0 + c1 t + c2 t^2, t = l/(N_L - 1),
                      lambda = sinh(a); Global / Segments / Curve.
 
-Readings where the paper is silent (each one is listed in the design doc):
+Readings where the paper is silent:
   * GQA: the window rows of a KV head are all n = G*W rows of the G query heads
     that share it; mu and sigma are taken over those n rows (sigma divisor n - 1,
     sigma = 0 when n = 1).

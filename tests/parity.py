@@ -1,6 +1,6 @@
 """Comparison of the CUDA path with the fp64 oracle (test helpers).
 
-Tolerances (derived in the design doc):
+Tolerances (the kernels compute A, mu and sigma in fp32 from bf16 inputs):
   mu:    |d| <= 1e-3 |mu_ref| + 1e-30                      (1e-3 relative)
   sigma: |d| <= 1e-3 |sigma_ref| + 1e-4 mu_ref + 1e-30     (sigma's error is carried by
                                                             the fp32 error of each A, which
