@@ -335,7 +335,9 @@ def run_ours(args):
     # min(B_l, L_r - W) + W rows per unit cross the host link, not the whole tensor.
     e2e = None
     if args.e2e_steps > 0:
-        chunks = args.e2e_chunks if N_L % args.e2e_chunks == 0 else 1
+        # layer chunks are contiguous views only for one request per plan
+        chunks = (args.e2e_chunks if args.e2e_chunks > 0 and N_L % args.e2e_chunks == 0
+                  and len(batch["seq_lens"]) == 1 else 1)
         Lc = N_L // chunks
         hq = q.cpu().pin_memory()
         hk = k.cpu().pin_memory()
