@@ -18,7 +18,9 @@
 //     When margins are requested the runner-up is brought up to date the same way.
 //  3. write the admitted positions ascending (and in admission order, with margins).
 // Values live in shared memory (C <= 32768); s~, corr and the inverse key norms in
-// the workspace; the admitted keys are read from K in global memory (L2).
+// the workspace; the first 96 admitted keys are staged in shared memory, later ones
+// are read from K in global memory (L2). A refresh applies the missing admissions in
+// groups of eight per pass over the candidate's row.
 #include "kve_internal.h"
 
 namespace kve {
@@ -26,6 +28,9 @@ namespace {
 
 constexpr int kAllThreads = 1024;
 constexpr int kAllWarps = kAllThreads / 32;
+constexpr int kAdmStage = 96;          // admitted keys staged in shared memory
+constexpr int kAdmStride = 17;         // uint4 per staged row (16 + 1 against bank conflicts)
+constexpr int kRefreshGroup = 8;       // missing admissions applied per pass over a candidate row
 
 __device__ __forceinline__ uint32_t ord_key_all(float f) {
   const uint32_t u = __float_as_uint(f + 0.0f);   // -0 -> +0
@@ -90,6 +95,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
   uint16_t* applied = reinterpret_cast<uint16_t*>(v + kMaxAllCand);  // [kMaxAllCand]
   int32_t* adm = reinterpret_cast<int32_t*>(applied + kMaxAllCand);  // [kMaxAllBudget]
   float* adm_inv = reinterpret_cast<float*>(adm + kMaxAllBudget);    // [kMaxAllBudget]
+  uint4* admk = reinterpret_cast<uint4*>(adm_inv + kMaxAllBudget);    // [kAdmStage][kAdmStride]
 
   // 1. pooled base score and its maximum
   float lmax = -INFINITY;
@@ -148,17 +154,45 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
   };
   rescan();
 
-  // candidate i brought up to date with admissions applied[i] .. t-1 by its owner
+  // candidate i brought up to date with admissions applied[i] .. t-1 by its owner,
+  // kRefreshGroup admissions per pass over the candidate's row (each dot keeps the
+  // element order of a plain loop); staged admitted keys come from shared memory
   auto refresh = [&](int i, int t) {
     const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kHeadDim);
     const float2 ci = cinv[i];
     const float inv_i = ci.y;
     float cmax = ci.x;
-    for (int a = applied[i]; a < t; ++a) {
-      const uint4* kj = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(adm[a]) * kHeadDim);
+    // admitted key a, chunk c: staged in shared memory or read from K
+    auto adm_chunk = [&](int a, int c) -> uint4 {
+      return a < kAdmStage ? admk[a * kAdmStride + c]
+                           : __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(adm[a]) * kHeadDim) + c);
+    };
+    int a0 = applied[i];
+    for (; a0 + kRefreshGroup <= t; a0 += kRefreshGroup) {
+      float dot[kRefreshGroup];
+#pragma unroll
+      for (int q = 0; q < kRefreshGroup; ++q) dot[q] = 0.f;
+      for (int c = 0; c < kHeadDim / 8; ++c) {
+        const uint4 x = __ldg(ki + c);
+        const uint32_t xa[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+        for (int q = 0; q < kRefreshGroup; ++q) {
+          const uint4 y = adm_chunk(a0 + q, c);
+          const uint32_t ya[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            dot[q] = fmaf(bf16_lo(xa[e]), bf16_lo(ya[e]), dot[q]);
+            dot[q] = fmaf(bf16_hi(xa[e]), bf16_hi(ya[e]), dot[q]);
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kRefreshGroup; ++q) cmax = fmaxf(cmax, dot[q] * inv_i * adm_inv[a0 + q]);
+    }
+    for (; a0 < t; ++a0) {
       float dot = 0.f;
       for (int c = 0; c < kHeadDim / 8; ++c) {
-        const uint4 x = __ldg(ki + c), y = __ldg(kj + c);
+        const uint4 x = __ldg(ki + c), y = adm_chunk(a0, c);
         const uint32_t xa[4] = {x.x, x.y, x.z, x.w}, ya[4] = {y.x, y.y, y.z, y.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -166,7 +200,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
           dot = fmaf(bf16_hi(xa[e]), bf16_hi(ya[e]), dot);
         }
       }
-      cmax = fmaxf(cmax, dot * inv_i * adm_inv[a]);
+      cmax = fmaxf(cmax, dot * inv_i * adm_inv[a0]);
     }
     cinv[i] = make_float2(cmax, inv_i);
     v[i] = fmaf(lambda2, cmax, st[i]);
@@ -199,6 +233,9 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
       v[bi] = -INFINITY;
       if (order) order[t] = bi;
     }
+    if (t < kAdmStage && tid < kHeadDim / 8)
+      admk[t * kAdmStride + tid] =
+          __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(bi) * kHeadDim) + tid);
     __syncthreads();
     if (tid == (bi % kAllThreads)) rescan();
     if (margins) {
@@ -251,7 +288,8 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
 
 cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {
   constexpr size_t smem = kMaxAllCand * (sizeof(float) + sizeof(uint16_t)) +
-                          kMaxAllBudget * (sizeof(int32_t) + sizeof(float));
+                          kMaxAllBudget * (sizeof(int32_t) + sizeof(float)) +
+                          kAdmStage * kAdmStride * sizeof(uint4);
   cudaError_t e = cudaFuncSetAttribute(select_all_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
