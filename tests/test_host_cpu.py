@@ -199,3 +199,24 @@ def test_every_candidate_plan_limits_without_gpu():
     with pytest.raises(K.KvEvictError) as e:
         big.select_profiles_workspace(2)
     assert e.value.status == K.KVE_EINVAL
+
+
+def test_gather_refuses_pageable_host_memory_without_gpu():
+    """kv_evict_gather reads k and v in place only from host memory the CUDA runtime
+    pinned: the binding refuses a pageable CPU tensor, and the C ABI returns
+    KVE_EINVAL for a pointer the runtime cannot classify (here: no GPU), both before
+    any launch."""
+    _need_lib()
+    torch = pytest.importorskip("torch")
+    from paper_2609_30738_gb300 import kv_evict as K
+    p = K.Plan(_spec(num_layers=1), [300])
+    k = torch.zeros((1, 8, 300, 128), dtype=torch.bfloat16)   # pageable
+    idx = torch.zeros((8, 64), dtype=torch.int32)
+    out = torch.zeros((8, 96, 128), dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        p.gather(k, k, idx, out, out)
+    if torch.cuda.is_available():
+        return   # the GPU suite checks the C ABI's refusal of pageable memory
+    buf = np.zeros(1 << 16, dtype=np.uint8)
+    ptr = buf.ctypes.data + (-buf.ctypes.data) % 16            # 16-byte aligned
+    assert K.library().kv_evict_gather(p._h, ptr, ptr, ptr, ptr, ptr, None) == K.KVE_EINVAL
