@@ -19,8 +19,9 @@
 //  3. write the admitted positions ascending (and in admission order, with margins).
 // Values live in shared memory (C <= 32768); s~, corr and the inverse key norms in
 // the workspace; the first 96 admitted keys are staged in shared memory, later ones
-// are read from K in global memory (L2). A refresh applies the missing admissions in
-// groups of eight per pass over the candidate's row.
+// are read from K in global memory (L2). For lambda2 <= 0 a warp refreshes its lanes'
+// stale bests together on the tensor cores; for lambda2 > 0 a thread applies the
+// missing admissions in groups of eight per pass over the candidate's row.
 #include "kve_internal.h"
 
 namespace kve {
@@ -206,11 +207,118 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
     v[i] = fmaf(lambda2, cmax, st[i]);
     applied[i] = static_cast<uint16_t>(t);
   };
-  // every owner whose best is stale brings it up to date, then takes its new best
+  // every owner whose best is stale brings it up to date, then takes its new best.
+  // A warp refreshes its lanes' stale bests together on the tensor cores: lane r's
+  // candidate row is row r of the A operand of mma.m16n8k16 (two m-tiles), the
+  // admitted keys a_lo .. t-1 form the B operand, 16 per pass (two n-tiles), where
+  // a_lo is the smallest count applied among the warp's stale bests; a dot against
+  // an admission already applied leaves the running maximum unchanged.
+  const uint32_t* kw32 = reinterpret_cast<const uint32_t*>(kb);          // 64 words per row
+  const uint32_t* admw = reinterpret_cast<const uint32_t*>(admk);        // 4 * kAdmStride words per row
   auto refresh_stale_bests = [&](int t) {
-    if (my_idx != 0xFFFFFFFFu && applied[my_idx] < t) {
-      refresh(static_cast<int>(my_idx), t);
-      rescan();
+    const bool stale = my_idx != 0xFFFFFFFFu && applied[my_idx] < t;
+    if (__any_sync(0xffffffffu, stale)) {
+      const int a_lo = static_cast<int>(__reduce_min_sync(
+          0xffffffffu, stale ? static_cast<uint32_t>(applied[my_idx]) : static_cast<uint32_t>(t)));
+      const int row = stale ? static_cast<int>(my_idx) : 0;      // row 0: a valid stand-in
+      const float2 ci = stale ? cinv[my_idx] : make_float2(0.f, 0.f);
+      float cm = ci.x;
+      const int g = lane >> 2, tq = lane & 3;
+      // rows g and g + 8 of m-tiles 0 and 1 belong to lanes 16m + 8hh + g
+      const uint32_t* ra[2][2];
+      float ir[2][2];
+#pragma unroll
+      for (int m = 0; m < 2; ++m)
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          const int src = 16 * m + 8 * hh + g;
+          ra[m][hh] = kw32 + static_cast<int64_t>(__shfl_sync(0xffffffffu, row, src)) * (kHeadDim / 2);
+          ir[m][hh] = __shfl_sync(0xffffffffu, ci.y, src);
+        }
+      for (int a0 = a_lo; a0 < t; a0 += 16) {
+        float d[2][2][4];
+#pragma unroll
+        for (int m = 0; m < 2; ++m)
+#pragma unroll
+          for (int n = 0; n < 2; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) d[m][n][e] = 0.f;
+        // column g of n-tile n is admission a0 + 8n + g (zero past t)
+        const uint32_t* rb[2];
+        bool bv[2];
+#pragma unroll
+        for (int n = 0; n < 2; ++n) {
+          const int an = a0 + 8 * n + g;
+          bv[n] = an < t;
+          rb[n] = !bv[n] ? kw32
+                         : (an < kAdmStage ? admw + an * (4 * kAdmStride)
+                                           : kw32 + static_cast<int64_t>(adm[an]) * (kHeadDim / 2));
+        }
+#pragma unroll
+        for (int s8 = 0; s8 < kHeadDim / 16; ++s8) {
+          uint32_t af[2][4];
+#pragma unroll
+          for (int m = 0; m < 2; ++m) {
+            af[m][0] = __ldg(ra[m][0] + 8 * s8 + tq);
+            af[m][1] = __ldg(ra[m][1] + 8 * s8 + tq);
+            af[m][2] = __ldg(ra[m][0] + 8 * s8 + tq + 4);
+            af[m][3] = __ldg(ra[m][1] + 8 * s8 + tq + 4);
+          }
+#pragma unroll
+          for (int n = 0; n < 2; ++n) {
+            const uint32_t b0 = bv[n] ? rb[n][8 * s8 + tq] : 0u;
+            const uint32_t b1 = bv[n] ? rb[n][8 * s8 + tq + 4] : 0u;
+#pragma unroll
+            for (int m = 0; m < 2; ++m) {
+              float* dd = d[m][n];
+              asm volatile(
+                  "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+                  "{%8,%9}, {%0,%1,%2,%3};"
+                  : "+f"(dd[0]), "+f"(dd[1]), "+f"(dd[2]), "+f"(dd[3])
+                  : "r"(af[m][0]), "r"(af[m][1]), "r"(af[m][2]), "r"(af[m][3]), "r"(b0), "r"(b1));
+            }
+          }
+        }
+        // element 2hh + e of d[m][n] is (row g + 8hh of m-tile m, column 2tq + e)
+        float rmax[2][2];
+#pragma unroll
+        for (int m = 0; m < 2; ++m) rmax[m][0] = rmax[m][1] = -INFINITY;
+#pragma unroll
+        for (int n = 0; n < 2; ++n)
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const int a = a0 + 8 * n + 2 * tq + e;
+            if (a < t) {
+              const float ia = adm_inv[a];
+#pragma unroll
+              for (int m = 0; m < 2; ++m)
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh)
+                  rmax[m][hh] = fmaxf(rmax[m][hh], d[m][n][2 * hh + e] * ir[m][hh] * ia);
+            }
+          }
+#pragma unroll
+        for (int m = 0; m < 2; ++m)
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            rmax[m][hh] = fmaxf(rmax[m][hh], __shfl_xor_sync(0xffffffffu, rmax[m][hh], 1));
+            rmax[m][hh] = fmaxf(rmax[m][hh], __shfl_xor_sync(0xffffffffu, rmax[m][hh], 2));
+          }
+        // lane 16m + 8hh + gg takes row (m, gg + 8hh) from lane 4gg
+        const int src = 4 * (lane & 7);
+        const float r00 = __shfl_sync(0xffffffffu, rmax[0][0], src);
+        const float r01 = __shfl_sync(0xffffffffu, rmax[0][1], src);
+        const float r10 = __shfl_sync(0xffffffffu, rmax[1][0], src);
+        const float r11 = __shfl_sync(0xffffffffu, rmax[1][1], src);
+        const float mine = (lane >> 4) ? ((lane >> 3) & 1 ? r11 : r10) : ((lane >> 3) & 1 ? r01 : r00);
+        cm = fmaxf(cm, mine);
+      }
+      if (stale) {
+        cinv[my_idx] = make_float2(cm, ci.y);
+        v[my_idx] = fmaf(lambda2, cm, st[my_idx]);
+        applied[my_idx] = static_cast<uint16_t>(t);
+        rescan();
+      }
     }
     __syncthreads();
   };
