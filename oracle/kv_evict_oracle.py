@@ -117,6 +117,13 @@ def base_score(mu_hat: np.ndarray, sigma_hat: np.ndarray, lambda1: float) -> np.
     return mu_hat + lambda1 * sigma_hat
 
 
+def pooled_base_score(mu: np.ndarray, sigma: np.ndarray, Lc: int, kernel: int,
+                      lambda1: float) -> np.ndarray:
+    """Section 3.1 pooling, then Eq. 2 without corr, over the candidates [0, Lc):
+    mu and sigma are max-pooled separately, then s_i = mu^_i + lambda1 sigma^_i."""
+    return base_score(max_pool(mu[:Lc], kernel), max_pool(sigma[:Lc], kernel), lambda1)
+
+
 def rank_desc(values: np.ndarray) -> np.ndarray:
     """Positions sorted by value descending, ties to the lower position."""
     return np.lexsort((np.arange(len(values)), -values))
@@ -232,9 +239,7 @@ def select_unit(mu: np.ndarray, sigma: np.ndarray, keys: np.ndarray, L: int, W: 
     cut_margin=s~ of the last pool member minus the first one left out).
     """
     Lc = L - W
-    mu_hat = max_pool(mu[:Lc], pool_kernel)
-    sigma_hat = max_pool(sigma[:Lc], pool_kernel)
-    s = base_score(mu_hat, sigma_hat, lambda1)
+    s = pooled_base_score(mu, sigma, Lc, pool_kernel, lambda1)
     C = Lc if candidate_factor == 0 else min(candidate_factor * B, Lc)
     ranked = rank_desc(s)
     pool = ranked[:C]

@@ -332,6 +332,161 @@ def test_budget_at_least_candidates_keeps_everything():
     np.testing.assert_array_equal(sel["indices"], np.arange(L - W))
 
 
+# --------------------------------------------------------------------------
+# Base score with lambda1 != 0: mu and sigma pooled separately (Section 3.1, Eq. 2)
+
+
+def _golden_pooled():
+    lines = [l.split() for l in open(os.path.join(GOLDEN, "pooled_base_score.txt"))
+             if l.strip() and not l.startswith("#")]
+    head = {p[0]: p[1:] for p in lines if p[0] != "case"}
+    kernel = int(head["kernel"][0])
+    mu = np.array([float(x) for x in head["mu"]])
+    sigma = np.array([float(x) for x in head["sigma"]])
+    cases = []
+    for p in lines:
+        if p[0] == "case":
+            i, j = p.index("s"), p.index("top2")
+            cases.append((float(p[1]), [float(x) for x in p[i + 1:j]], [int(x) for x in p[j + 1:]]))
+    return kernel, mu, sigma, cases
+
+
+def test_pooled_base_score_worked_example():
+    """Hand-worked s = mu^ + lambda1 sigma^ (separate pooling) for lambda1 in
+    {0.5, -0.3, 2}, and the top 2 by the whole-unit selection at lambda2 = 0."""
+    kernel, mu, sigma, cases = _golden_pooled()
+    Lc = len(mu)
+    W = 1
+    keys = np.eye(Lc + W, 4)            # irrelevant at lambda2 = 0
+    mu_all = np.append(mu, 0.0)         # the window token (not a candidate)
+    sg_all = np.append(sigma, 0.0)
+    for lam1, s_ref, top2 in cases:
+        s = O.pooled_base_score(mu_all, sg_all, Lc, kernel, lam1)
+        np.testing.assert_allclose(s, s_ref, rtol=0, atol=1e-15)
+        sel = O.select_unit(mu_all, sg_all, keys, Lc + W, W, 2, lam1, 0.0, pool_kernel=kernel)
+        assert [st["pick"] for st in sel["steps"]] == top2
+        np.testing.assert_allclose(sel["s_tilde"], np.array(s_ref) / max(s_ref), rtol=1e-15)
+
+
+def _pooled_reference(mu, sigma, Lc, k, lam1, B, eps=1e-12):
+    """Built outside the oracle: scipy's max filter on mu and on sigma separately,
+    then a plain sort (value descending, then position ascending)."""
+    mh = scipy.ndimage.maximum_filter1d(mu[:Lc], size=k, mode="nearest")
+    sh = scipy.ndimage.maximum_filter1d(sigma[:Lc], size=k, mode="nearest")
+    s = mh + lam1 * sh
+    order = sorted(range(Lc), key=lambda i: (-s[i], i))
+    return s / max(max(s), eps), order[:B]
+
+
+@pytest.mark.parametrize("lam1", [0.5, -0.3, 2.0])
+@pytest.mark.parametrize("k", [3, 7])
+def test_pooled_base_score_lambda1_matches_scipy(lam1, k):
+    """lambda2 = 0 makes the greedy a sort, so the whole-unit selection is the top-B
+    of the pooled base score; with lambda1 != 0, how sigma is pooled and weighted
+    decides the set. s~ and the admissions match the reference built above."""
+    L, W, B = 160, 8, 12
+    for seed in (21, 22):
+        mu, sigma, k_ = _unit(seed, L, W)
+        sel = O.select_unit(mu, sigma, k_, L, W, B, lam1, 0.0, pool_kernel=k)
+        st_ref, top = _pooled_reference(mu, sigma, L - W, k, lam1, B)
+        np.testing.assert_allclose(sel["s_tilde"], st_ref, rtol=1e-13, atol=1e-300)
+        assert [s["pick"] for s in sel["steps"]] == top
+
+
+def _joint_pooling(mu, sigma, Lc, kernel, lambda1):
+    return O.max_pool(mu[:Lc] + lambda1 * sigma[:Lc], kernel)
+
+
+@pytest.mark.parametrize("bad", [
+    ("pool", _joint_pooling),                                   # s = maxpool(mu + l1 sigma)
+    ("base", lambda m, s, l1: m + l1 * s * s),                  # s = mu + l1 sigma^2
+    ("base", lambda m, s, l1: m + 0.5 * l1 * s),                # s = mu + l1 sigma / 2
+])
+def test_planted_base_score_bugs_are_caught(monkeypatch, bad):
+    """Each plausible mistake in the pooled base score fails a pin above."""
+    where, fn = bad
+    monkeypatch.setattr(O, "pooled_base_score" if where == "pool" else "base_score", fn)
+    failed = 0
+    try:
+        test_pooled_base_score_worked_example()
+    except AssertionError:
+        failed += 1
+    for lam1 in (0.5, -0.3, 2.0):
+        try:
+            test_pooled_base_score_lambda1_matches_scipy(lam1, 7)
+        except AssertionError:
+            failed += 1
+    assert failed >= 2
+
+
+# --------------------------------------------------------------------------
+# Forced replay (the branch parity checking runs through on every near-tie swap)
+
+
+def _brute_value(i, prior, s_tilde, keys, lam2):
+    """s~_i + lambda2 * corr(i, prior) with corr from Eq. 4 by plain loops."""
+    c = 0.0
+    for j in prior:
+        a, b = keys[i], keys[j]
+        na = math.sqrt(sum(x * x for x in a))
+        nb = math.sqrt(sum(x * x for x in b))
+        cs = 0.0 if na == 0 or nb == 0 else sum(x * y for x, y in zip(a, b)) / (na * nb)
+        c = max(c, cs)
+    return s_tilde[i] + lam2 * c
+
+
+def _forced_case():
+    """A unit where the forced sequence takes a position outside the top-4B pool,
+    with that key a near-duplicate of a pool member, so its corr and the corr it
+    adds to others are both far from 0."""
+    L, W, B = 200, 8, 6
+    rng = np.random.default_rng(31)
+    mu, sigma, keys = _unit(31, L, W)
+    sel = O.select_unit(mu, sigma, keys, L, W, B, 0.5, -0.6)
+    pool = [int(x) for x in sel["pool"]]
+    ranked = O.rank_desc(sel["s_tilde"])
+    outside = int(ranked[len(pool) + 3])                   # not in the pool
+    keys = keys.copy()
+    mate = pool[5]
+    keys[outside] = keys[mate] + 0.05 * rng.standard_normal(keys.shape[1])
+    first = [int(s["pick"]) for s in O.select_unit(mu, sigma, keys, L, W, B, 0.5, -0.6)["steps"]]
+    follow = first[:2] + [outside] + first[2:5]
+    return mu, sigma, keys, L, W, B, pool, outside, mate, follow
+
+
+def test_forced_replay_out_of_pool_pick():
+    """follow = the oracle's own picks with one position from outside the pool forced
+    in at step 2: every step's v_pick, v_best, best and margin equal brute force over
+    the grown admitted set (the forced key counts in later corr, Eq. 4)."""
+    mu, sigma, keys, L, W, B, pool, outside, mate, follow = _forced_case()
+    lam2 = -0.6
+    ref = O.select_unit(mu, sigma, keys, L, W, B, 0.5, lam2, follow=follow)
+    st = ref["s_tilde"]
+    assert outside not in pool
+    assert [s["pick"] for s in ref["steps"]] == follow
+    taken = []
+    for t, step in enumerate(ref["steps"]):
+        assert abs(step["v_pick"] - _brute_value(step["pick"], taken, st, keys, lam2)) < 1e-12
+        rest = [i for i in pool if i not in taken]
+        vals = sorted(((-_brute_value(i, taken, st, keys, lam2), i) for i in rest))
+        assert step["best"] == vals[0][1]
+        assert abs(step["v_best"] + vals[0][0]) < 1e-12
+        assert abs(step["margin"] - (vals[1][0] - vals[0][0])) < 1e-12
+        taken.append(step["pick"])
+    # the forced key is a near-duplicate of `mate`: after step 2 mate's corr is ~1
+    t_after = 3
+    if mate not in follow[:t_after]:
+        v_mate = _brute_value(mate, follow[:t_after], st, keys, lam2)
+        assert v_mate < st[mate] + lam2 * 0.9
+
+
+def test_planted_forced_replay_bug_is_caught(monkeypatch):
+    """Admitting an out-of-pool position with corr = 0 instead of Eq. 4 fails the pin."""
+    monkeypatch.setattr(O, "corr", lambda i, S, keys: 0.0)
+    with pytest.raises(AssertionError):
+        test_forced_replay_out_of_pool_pick()
+
+
 def test_gather_rows_and_zero_tail():
     rng = np.random.default_rng(15)
     L, W, B, d = 20, 4, 8, 6
