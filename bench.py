@@ -1,16 +1,20 @@
 """Benchmark of the end-of-prefill diversified KV-eviction step on GB300.
 
-One step = the whole path for one request of the Mistral-7B-shaped workload
-"mistral-32layer-L32768-B64": 32 layers x 8 KV heads (256 units), prefix 32768,
-window 32, budget 64, lambda = (0.5, -0.5): score (window attention, mu, sigma),
-select (pooling, top-4B, greedy MMR) and gather (compact K/V cache).
+One step = the whole path for one call of a Mistral-7B-shaped workload: score
+(window attention, mu, sigma), select (pooling, top-4B, greedy MMR) and gather
+(compact K/V cache). The default workload is "mistral-32layer-L32768-B64": one
+request of 32 layers x 8 KV heads (256 units), prefix 32768, window 32, budget 64,
+lambda = (0.5, -0.5). --workload names any of the full-size workloads.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload NAME]
 
-N > 1 runs under torchrun, one rank per GPU; every rank evicts its own request
-(weak scaling, no collective on the data path). Rank 0 prints one JSON line.
---impl reference times the fp64 CPU oracle (the only reference this path has) on
-a bounded sample of the same workload on the host cores.
+N > 1 runs under torchrun, one rank per GPU, with no collective on the data path.
+A one-request workload gives every rank its own request (weak scaling); the
+16-request batch is split across the ranks by prefix tokens (strong scaling).
+Rank 0 prints one JSON line. --impl reference times the fp64 CPU oracle (the only
+reference this path has) on a bounded sample of the same workload on the host
+cores.
 """
 
 from __future__ import annotations
@@ -31,6 +35,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 WORKLOAD = "mistral-32layer-L32768-B64"
+BENCH_WORKLOADS = ("mistral-32layer-L8192", "mistral-32layer-L32768-B32", "mistral-32layer-L32768-B64",
+                   "mistral-32layer-L32768-B128", "mistral-32layer-L16384-segments",
+                   "mistral-32layer-ragged16")
 METRIC = "eviction-step ms/request (32 layers) & prefix tok/s; % of HBM roofline"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
@@ -79,6 +86,46 @@ def _max_over_ranks(x, world, device):
 def _job_tok_s(world, prefix_len, step_s):
     """Whole-job throughput: every rank evicts one request of prefix_len tokens per step."""
     return world * prefix_len / step_s
+
+
+def _rank_requests(spec, world, rank):
+    """(request ids this rank evicts, scaling). A one-request workload: every rank
+    its own request (id = rank), weak scaling. A batch: the batch's requests split
+    across the ranks by prefix tokens, strong scaling."""
+    from paper_2609_30738_gb300.workloads import partition_requests
+    if len(spec["seq_lens"]) == 1:
+        return [rank], "weak"
+    return partition_requests(spec["seq_lens"], world)[rank], "strong"
+
+
+def _config(name, spec, world):
+    """The `config` object of both arms' JSON lines (identical for the same workload
+    and number of GPUs)."""
+    seq = spec["seq_lens"]
+    scaling = "weak" if len(seq) == 1 else "strong"
+    return {"workload": name, "parallelism": f"{scaling} x{world} (requests per rank, no collective)",
+            "requests_per_step_job": world if scaling == "weak" else len(seq), "layers": spec["num_layers"], "kv_heads": spec["num_kv_heads"],
+            "q_heads": spec["num_q_heads"], "head_dim": spec["head_dim"],
+            "prefix_len": seq[0] if len(seq) == 1 else f"{len(seq)} requests, {min(seq)}-{max(seq)}",
+            "tokens_per_call": sum(seq), "window": spec["window"], "budget": spec["budget"],
+            "lambdas": list(spec["lambdas"][:1]) + [str(x) for x in spec["lambdas"][1:]],
+            "pool_kernel": spec["pool_kernel"],
+            "l2": "inputs larger than L2 (the K read per step exceeds 129 MB)"}
+
+
+def _algorithmic_bytes(spec, seq, layer_budgets):
+    """Algorithmic bytes of one step (bytes that must cross HBM): K read once
+    (L d 2 per unit) by the score kernel; K and V rows gathered (min(B_l, L - W) + W
+    rows read per unit and B + W rows written, K and V). Secondary traffic, not
+    counted: the window queries (n d 2 per unit) and the mu / sigma writes (8 L)."""
+    N_L, Hkv, W, B, d = (spec["num_layers"], spec["num_kv_heads"], spec["window"], spec["budget"],
+                         spec["head_dim"])
+    n = spec["num_q_heads"] // Hkv * W
+    k_read = sum(N_L * Hkv * L * d * 2 for L in seq)
+    gather = sum(Hkv * 2 * ((min(layer_budgets[l], L - W) + W) + (B + W)) * d * 2
+                 for L in seq for l in range(N_L))
+    secondary = sum(N_L * Hkv * (n * d * 2 + 8 * L) for L in seq)
+    return k_read, gather, secondary
 
 
 class ClockSampler:
@@ -160,7 +207,7 @@ def _oracle_unit(u):
 class OraclePool:
     """Spawned worker processes (one BLAS thread each) over a memory-mapped sample."""
 
-    def __init__(self, spec, sample, workers):
+    def __init__(self, spec, sample, workers, sample_len, lam):
         import multiprocessing as mp
         import tempfile
         for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
@@ -176,7 +223,7 @@ class OraclePool:
             mm[i] = np.concatenate([q.reshape(-1), k.reshape(-1)])
         mm.flush()
         del mm
-        meta = (spec["seq_lens"][0], spec["window"], G, spec["budget"], 0.5, -0.5)
+        meta = (sample_len, spec["window"], G, spec["budget"], lam[0], lam[1])
         self.n = n
         self.pool = mp.get_context("spawn").Pool(
             workers, initializer=_oracle_init, initargs=(self.path, n, q_shape, k_shape, meta))
@@ -198,7 +245,8 @@ class OraclePool:
 
 
 def _oracle_sample_from_host(spec, n_units, seed):
-    """(q_bits, k_bits) of the first n_units units, generated on the CPU."""
+    """(q_bits, k_bits) of the first n_units units (layer-major, then KV head) of
+    request 0, generated on the CPU."""
     import torch
     from paper_2609_30738_gb300 import synth
     from tests.parity import to_bits
@@ -216,17 +264,29 @@ def _oracle_sample_from_host(spec, n_units, seed):
     return out
 
 
+def _layer0_lambdas(spec):
+    from oracle import kv_evict_oracle as O
+    from paper_2609_30738_gb300.workloads import lambda_arrays
+    l1, l2 = lambda_arrays(spec, O.depth_profile)
+    return float(l1[0]), float(l2[0])
+
+
 def run_reference(args):
-    """--impl reference: the fp64 oracle on the host cores, bounded sample per step."""
+    """--impl reference: the fp64 oracle on the host cores. A step is one pass over a
+    bounded sample (one unit per host core) of request 0 of the workload; the line
+    reports the measured wall time of that pass as ms_per_step and the throughput
+    of the sample (its share of the request's prefix tokens per second)."""
     world, rank, _ = _dist()
     if rank != 0:
         return
     from paper_2609_30738_gb300.workloads import WORKLOADS
-    spec = WORKLOADS[WORKLOAD]
+    name = args.workload
+    spec = WORKLOADS[name]
     cores = os.cpu_count() or 1
     n_units = cores          # one unit per host core and step
+    L = spec["seq_lens"][0]
     sample = _oracle_sample_from_host(spec, n_units, 2609)
-    pool = OraclePool(spec, sample, cores)
+    pool = OraclePool(spec, sample, cores, L, _layer0_lambdas(spec))
     try:
         for _ in range(args.warmup):
             pool.run()
@@ -234,18 +294,20 @@ def run_reference(args):
     finally:
         pool.close()
     step_s = sum(times) / len(times)
-    units_total = spec["num_layers"] * spec["num_kv_heads"]
-    L = spec["seq_lens"][0]
-    tok_s = L * (n_units / units_total) / step_s
-    ms_req = step_s * 1e3 * units_total / n_units
+    units_req = spec["num_layers"] * spec["num_kv_heads"]
+    tok_s = L * (n_units / units_req) / step_s
+    desc = (f"{n_units} of the {units_req} units of request 0 (L = {L}; score + select, one unit "
+            f"per worker) per step; measured wall {step_s * 1e3:.1f} ms per step")
     line = {"impl": "reference", "metric": METRIC, "value": tok_s, "unit": "prefix tok/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": ms_req, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "sample_units": n_units},
+            "ms_per_step": step_s * 1e3, "higher_is_better": True,
+            "scaling": "weak" if len(spec["seq_lens"]) == 1 else "strong",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded Mistral-7B-shaped K/Q)",
+            "config": _config(name, spec, world),
+            "sample_units_per_step": n_units,
+            "extrapolated_ms_per_request": step_s * 1e3 * units_req / n_units,
             "cpu_baseline": {"value": tok_s, "unit": "prefix tok/s", "cores": cores, "kind": "oracle",
-                             "sample": f"{n_units} of 256 units (score + select) per step, "
-                                       "extrapolated to the 256-unit request"},
+                             "sample": desc},
             "e2e": {"value": tok_s, "unit": "prefix tok/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -266,33 +328,39 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
-    spec = WORKLOADS[WORKLOAD]
+    name = args.workload
+    full = WORKLOADS[name]
+    reqs, scaling = _rank_requests(full, world, rank)
+    spec = dict(full, seq_lens=[full["seq_lens"][0]] * len(reqs) if len(full["seq_lens"]) == 1
+                else [full["seq_lens"][r] for r in reqs])
     if args.layers:
         spec = dict(spec, num_layers=args.layers)
-    L = spec["seq_lens"][0]
     W, B, d = spec["window"], spec["budget"], spec["head_dim"]
     N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
-    units = N_L * Hkv
+    seq = spec["seq_lens"]
+    tokens = sum(seq)                      # prefix tokens this rank evicts per step
+    # requests per step over the job (weak: one per rank; strong: the batch)
+    job_requests = world if scaling == "weak" else len(full["seq_lens"])
 
-    # inputs resident in HBM: each rank evicts its own request (seeded by rank)
-    batch = synth.make_batch(spec, seed=2609 + rank, device=dev)
-    q, k, v = batch["q_win"], batch["k"], batch["v"]
-    plan = K.Plan(spec, batch["seq_lens"])
-    bufs = K.Buffers(plan, device=dev, with_trace=False)
+    # inputs resident in HBM; a batch's subset keeps its requests' seeds
+    batch = synth.make_batch(spec, seed=2609, device=dev, request_ids=reqs) if reqs else None
     lam1, lam2 = lambda_arrays(spec, K.profile)
     stream = torch.cuda.Stream(device=dev)
+    if batch is not None:
+        q, k, v = batch["q_win"], batch["k"], batch["v"]
+        plan = K.Plan(spec, batch["seq_lens"])
+        bufs = K.Buffers(plan, device=dev, with_trace=False)
 
-    def step():
-        K.run_step(plan, bufs, q, k, v, lam1, lam2, stream=stream)
+        def step():
+            K.run_step(plan, bufs, q, k, v, lam1, lam2, stream=stream)
 
-    # correctness of the timed configuration: device status after a first step
-    with torch.cuda.stream(stream):
-        step()
-    if plan.status(bufs.ws, stream) != K.KVE_OK:
-        raise RuntimeError("device-side wait timed out")
-
-    for _ in range(args.warmup):
-        step()
+        # correctness of the timed configuration: device status after a first step
+        with torch.cuda.stream(stream):
+            step()
+        if plan.status(bufs.ws, stream) != K.KVE_OK:
+            raise RuntimeError("device-side wait timed out")
+        for _ in range(args.warmup):
+            step()
     stream.synchronize()
 
     sampler = ClockSampler(local) if rank == 0 else None
@@ -308,7 +376,7 @@ def run_ours(args):
     if sampler:
         sampler.mark("t0")
     t0.record(stream)
-    for i in range(args.steps):
+    for i in range(args.steps if batch is not None else 0):
         ev[i][0].record(stream)
         plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws, stream)
         ev[i][1].record(stream)
@@ -321,125 +389,69 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     elapsed = t0.elapsed_time(t1) / 1e3
-    score_s = sum(a.elapsed_time(b) for a, b in ev) / 1e3 / args.steps
+    score_s = (sum(a.elapsed_time(b) for a, b in ev) / 1e3 / args.steps) if batch is not None else 0.0
     clocks = sampler.stop() if sampler else None
-    if plan.status(bufs.ws, stream) != K.KVE_OK:
+    if batch is not None and plan.status(bufs.ws, stream) != K.KVE_OK:
         raise RuntimeError("device-side wait timed out in the timed region")
     elapsed = _max_over_ranks(elapsed, world, dev)
 
     # end to end through the public API with host buffers (pinned), copies inside.
-    # The request is evicted in chunks of layers, one plan per chunk: the copy stream
-    # brings in chunk c + 1 while the compute stream scores, selects and gathers chunk
-    # c (every array is layer-major for one request, so a chunk is a contiguous view).
-    # V stays in pinned host memory: the gather reads the kept rows in place, so
-    # min(B_l, L_r - W) + W rows per unit cross the host link, not the whole tensor.
+    # A one-request call is evicted in chunks of layers, one plan per chunk: the copy
+    # stream brings in chunk c + 1 while the compute stream scores, selects and
+    # gathers chunk c (every array is layer-major for one request, so a chunk is a
+    # contiguous view). V stays in pinned host memory: the gather reads the kept rows
+    # in place, so min(B_l, L_r - W) + W rows per unit cross the host link, not the
+    # whole tensor.
     e2e = None
     if args.e2e_steps > 0:
-        # layer chunks are contiguous views only for one request per plan
-        chunks = (args.e2e_chunks if args.e2e_chunks > 0 and N_L % args.e2e_chunks == 0
-                  and len(batch["seq_lens"]) == 1 else 1)
-        Lc = N_L // chunks
-        hq = q.cpu().pin_memory()
-        hk = k.cpu().pin_memory()
-        hv = v.cpu().pin_memory()
-        o_idx = torch.empty_like(bufs.indices, device="cpu").pin_memory()
-        o_k = torch.empty_like(bufs.k_out, device="cpu").pin_memory()
-        o_v = torch.empty_like(bufs.v_out, device="cpu").pin_memory()
-        dq, dk = torch.empty_like(q), torch.empty_like(k)
-        cplan = K.Plan(dict(spec, num_layers=Lc), batch["seq_lens"])
-        cws = torch.empty(cplan.workspace_bytes, dtype=torch.uint8, device=dev)
-        mu_c = bufs.mu.view(chunks, -1)
-        sg_c = bufs.sigma.view(chunks, -1)
-        idx_c = bufs.indices.view(chunks, Lc * Hkv, -1)
-        ko_c = bufs.k_out.view(chunks, Lc * Hkv, *bufs.k_out.shape[1:])
-        vo_c = bufs.v_out.view(chunks, Lc * Hkv, *bufs.v_out.shape[1:])
-        copy_stream = torch.cuda.Stream(device=dev)
-        arrived = [torch.cuda.Event() for _ in range(chunks)]
-        v_rows = sum(Hkv * (min(plan.layer_budgets[l], Lr - W) + W)
-                     for Lr in plan.seq_lens for l in range(N_L))
-        v_read = v_rows * d * hv.element_size()
-
-        def e2e_step():
-            copy_stream.wait_stream(stream)    # the previous step has finished with dq, dk
-            with torch.cuda.stream(copy_stream):
-                for c in range(chunks):
-                    dq[c * Lc:(c + 1) * Lc].copy_(hq[c * Lc:(c + 1) * Lc], non_blocking=True)
-                    dk[c * Lc:(c + 1) * Lc].copy_(hk[c * Lc:(c + 1) * Lc], non_blocking=True)
-                    arrived[c].record(copy_stream)
-            for c in range(chunks):
-                ls = slice(c * Lc, (c + 1) * Lc)
-                stream.wait_event(arrived[c])
-                cplan.score(dq[ls], dk[ls], mu_c[c], sg_c[c], cws, stream)
-                cplan.select(mu_c[c], sg_c[c], dk[ls], lam1[ls], lam2[ls], idx_c[c], cws, None, None,
-                             stream)
-                cplan.gather(dk[ls], hv[ls], idx_c[c], ko_c[c], vo_c[c], stream)
-            with torch.cuda.stream(stream):
-                o_idx.copy_(bufs.indices, non_blocking=True)
-                o_k.copy_(bufs.k_out, non_blocking=True)
-                o_v.copy_(bufs.v_out, non_blocking=True)
-
-        for _ in range(2):                     # first touches of the pinned buffers
-            e2e_step()
-        stream.synchronize()
-        if cplan.status(cws, stream) != K.KVE_OK:
-            raise RuntimeError("device-side wait timed out in the end-to-end step")
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        if world > 1:
-            dist.barrier()
-        copy_stream.wait_stream(stream)
-        a.record(copy_stream)
-        for _ in range(args.e2e_steps):
-            e2e_step()
-        b.record(stream)
-        torch.cuda.synchronize()
-        if cplan.status(cws, stream) != K.KVE_OK:
-            raise RuntimeError("device-side wait timed out in the end-to-end step")
-        e2e_s = a.elapsed_time(b) / 1e3 / args.e2e_steps
+        e2e_s, h2d, d2h, chunks = 0.0, 0, 0, 1
+        if batch is not None:
+            e2e_s, h2d, d2h, chunks = _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream, dev, world)
+        elif world > 1:
+            dist.barrier()                 # the one in _e2e, for a rank without requests
         e2e_s = _max_over_ranks(e2e_s, world, dev)
-        h2d = sum(x.numel() * x.element_size() for x in (hq, hk)) + v_read
-        d2h = sum(x.numel() * x.element_size() for x in (o_idx, o_k, o_v))
-        e2e = {"value": _job_tok_s(world, L, e2e_s), "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
+        job_tokens = tokens * world if scaling == "weak" else sum(full["seq_lens"])
+        e2e = {"value": job_tokens / e2e_s, "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "layer_chunks": chunks,
                "v": "read in place from pinned host memory by the gather (kept rows only)"}
-        del hq, hk, hv, dq, dk
 
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
         return
 
-    # roofline of the dominant kernel (score): algorithmic bytes per launch
-    n_rows = spec["num_q_heads"] // Hkv * W
-    score_bytes = units * (L * d * 2 + n_rows * d * 2 + 2 * 4 * L)
-    gather_bytes = units * 2 * 2 * (B + W) * d * 2
+    # roofline: algorithmic bytes (K read + K/V gathered) over the measured HBM peak;
+    # the dominant kernel (score) reads K
+    k_read, gather_bytes, secondary = _algorithmic_bytes(spec, seq, plan.layer_budgets)
     peak, peak_kind = _peaks()
-    achieved = score_bytes / score_s / 1e9
+    achieved = k_read / score_s / 1e9
     traffic = (SCORE_TRAFFIC["bytes_per_launch"]
-               if SCORE_TRAFFIC["source_sha256"] == _score_source_sha() else None)
+               if (SCORE_TRAFFIC["source_sha256"] == _score_source_sha() and name == WORKLOAD
+                   and not args.layers) else None)
 
     cpu = None
     if world == 1 and args.cpu_units > 0:
         cpu = cpu_baseline_from_device(spec, batch, args.cpu_units)
 
     step_s = elapsed / args.steps
-    line = {"metric": METRIC, "value": _job_tok_s(world, L, step_s), "unit": "prefix tok/s", "n_gpus": world,
+    job_tokens = tokens * world if scaling == "weak" else sum(full["seq_lens"])
+    config = _config(name, full, world)
+    if args.layers:
+        config["workload"] = f"{name} ({N_L} layers)"
+    line = {"metric": METRIC, "value": job_tokens / step_s, "unit": "prefix tok/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "higher_is_better": True, "scaling": scaling, "vs_baseline": None,
             "dtype": "bf16xbf16->f32", "data": "synthetic (seeded Mistral-7B-shaped K/V/Q)",
-            "config": {"workload": WORKLOAD if not args.layers else f"{WORKLOAD} ({N_L} layers)",
-                       "layers": N_L, "kv_heads": Hkv,
-                       "q_heads": spec["num_q_heads"], "head_dim": d, "prefix_len": L,
-                       "window": W, "budget": B, "lambda1": 0.5, "lambda2": -0.5,
-                       "pool_kernel": spec["pool_kernel"], "requests_per_gpu": 1,
-                       "l2": "inputs larger than L2 (2.15 GB of K read per step)"},
-            "ms_per_request": step_s * 1e3,
-            "hbm_roofline_frac_step": (score_bytes + gather_bytes) / step_s / 1e9 / peak,
+            "config": config,
+            "ms_per_request": step_s * 1e3 * world / job_requests,
+            "hbm_roofline_frac_step": (k_read + gather_bytes) / step_s / 1e9 / peak,
+            "algorithmic_bytes_step": {"k_read": k_read, "kv_gathered": gather_bytes},
             "score_kernel_ms": score_s * 1e3,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
                          "peak_source": peak_kind, "kernel": "kve score_kernel",
-                         "algorithmic_bytes_per_launch": score_bytes},
+                         "algorithmic_bytes_per_launch": k_read,
+                         "secondary_bytes_per_launch": secondary},
             "gpu_launches": 3 * args.steps,
             "clocks": clocks, "cpu_baseline": cpu, "e2e": e2e}
     print(json.dumps(line), flush=True)
@@ -447,28 +459,106 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream, dev, world):
+    """End-to-end step through the public API: seconds per step, H2D and D2H bytes
+    per step, layer chunks."""
+    import torch
+    import torch.distributed as dist
+    from paper_2609_30738_gb300 import kv_evict as K
+    q, k, v = batch["q_win"], batch["k"], batch["v"]
+    W, d = spec["window"], spec["head_dim"]
+    N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
+    # layer chunks are contiguous views only for one request per plan
+    chunks = (args.e2e_chunks if args.e2e_chunks > 0 and N_L % args.e2e_chunks == 0
+              and len(batch["seq_lens"]) == 1 else 1)
+    Lc = N_L // chunks
+    hq = q.cpu().pin_memory()
+    hk = k.cpu().pin_memory()
+    hv = v.cpu().pin_memory()
+    o_idx = torch.empty_like(bufs.indices, device="cpu").pin_memory()
+    o_k = torch.empty_like(bufs.k_out, device="cpu").pin_memory()
+    o_v = torch.empty_like(bufs.v_out, device="cpu").pin_memory()
+    dq, dk = torch.empty_like(q), torch.empty_like(k)
+    cplan = K.Plan(dict(spec, num_layers=Lc), batch["seq_lens"])
+    cws = torch.empty(cplan.workspace_bytes, dtype=torch.uint8, device=dev)
+    mu_c = bufs.mu.view(chunks, -1)
+    sg_c = bufs.sigma.view(chunks, -1)
+    idx_c = bufs.indices.view(chunks, -1, bufs.indices.shape[1])
+    ko_c = bufs.k_out.view(chunks, -1, *bufs.k_out.shape[1:])
+    vo_c = bufs.v_out.view(chunks, -1, *bufs.v_out.shape[1:])
+    copy_stream = torch.cuda.Stream(device=dev)
+    arrived = [torch.cuda.Event() for _ in range(chunks)]
+    v_rows = sum(Hkv * (min(plan.layer_budgets[l], Lr - W) + W)
+                 for Lr in plan.seq_lens for l in range(N_L))
+    v_read = v_rows * d * hv.element_size()
+
+    def e2e_step():
+        copy_stream.wait_stream(stream)    # the previous step has finished with dq, dk
+        with torch.cuda.stream(copy_stream):
+            for c in range(chunks):
+                dq[c * Lc:(c + 1) * Lc].copy_(hq[c * Lc:(c + 1) * Lc], non_blocking=True)
+                dk[c * Lc:(c + 1) * Lc].copy_(hk[c * Lc:(c + 1) * Lc], non_blocking=True)
+                arrived[c].record(copy_stream)
+        for c in range(chunks):
+            ls = slice(c * Lc, (c + 1) * Lc)
+            stream.wait_event(arrived[c])
+            cplan.score(dq[ls], dk[ls], mu_c[c], sg_c[c], cws, stream)
+            cplan.select(mu_c[c], sg_c[c], dk[ls], lam1[ls], lam2[ls], idx_c[c], cws, None, None,
+                         stream)
+            cplan.gather(dk[ls], hv[ls], idx_c[c], ko_c[c], vo_c[c], stream)
+        with torch.cuda.stream(stream):
+            o_idx.copy_(bufs.indices, non_blocking=True)
+            o_k.copy_(bufs.k_out, non_blocking=True)
+            o_v.copy_(bufs.v_out, non_blocking=True)
+
+    for _ in range(2):                     # first touches of the pinned buffers
+        e2e_step()
+    stream.synchronize()
+    if cplan.status(cws, stream) != K.KVE_OK:
+        raise RuntimeError("device-side wait timed out in the end-to-end step")
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    copy_stream.wait_stream(stream)
+    a.record(copy_stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    if cplan.status(cws, stream) != K.KVE_OK:
+        raise RuntimeError("device-side wait timed out in the end-to-end step")
+    e2e_s = a.elapsed_time(b) / 1e3 / args.e2e_steps
+    h2d = sum(x.numel() * x.element_size() for x in (hq, hk)) + v_read
+    d2h = sum(x.numel() * x.element_size() for x in (o_idx, o_k, o_v))
+    return e2e_s, h2d, d2h, chunks
+
+
 def cpu_baseline_from_device(spec, batch, n_units):
-    """Oracle on the first n_units units of the device-resident inputs."""
+    """Oracle on the first n_units units (request 0) of the device-resident inputs:
+    the measured wall time of that sample, and the throughput it implies."""
     from tests.parity import to_bits
     G = spec["num_q_heads"] // spec["num_kv_heads"]
-    W, Hkv = spec["window"], spec["num_kv_heads"]
+    W, Hkv, L = spec["window"], spec["num_kv_heads"], spec["seq_lens"][0]
+    units_req = spec["num_layers"] * Hkv
+    n_units = min(n_units, units_req)
     sample = []
     for u in range(n_units):
         layer, h = divmod(u, Hkv)
         sample.append((to_bits(batch["q_win"][layer, 0, h * G:(h + 1) * G]).reshape(G * W, -1),
-                       to_bits(batch["k"][layer, h])))
+                       to_bits(batch["k"][layer, h, :L])))
     cores = min(os.cpu_count() or 1, n_units)
-    pool = OraclePool(spec, sample, cores)
+    pool = OraclePool(spec, sample, cores, L, _layer0_lambdas(spec))
     try:
         wall = pool.run()
     finally:
         pool.close()
-    units_total = spec["num_layers"] * Hkv
-    L = spec["seq_lens"][0]
-    return {"value": L * (n_units / units_total) / wall, "unit": "prefix tok/s", "cores": cores,
+    return {"value": L * (n_units / units_req) / wall, "unit": "prefix tok/s", "cores": cores,
             "kind": "oracle",
-            "sample": f"{n_units} of {units_total} units (score + select), wall {wall:.1f} s on "
-                      f"{cores} worker processes, extrapolated to the whole request"}
+            "sample": f"{n_units} of the {units_req} units of request 0 (L = {L}; score + select) "
+                      f"on {cores} worker processes",
+            "sample_wall_s": wall,
+            "extrapolated_ms_per_request": wall * 1e3 * units_req / n_units}
 
 
 def main():
@@ -477,6 +567,7 @@ def main():
     ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=BENCH_WORKLOADS, default=WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="layer chunks of the end-to-end step (copy of chunk c+1 beside compute of c)")

@@ -159,7 +159,9 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu,
  * what kv_evict_select selects with lambda1 + p*N_L and lambda2 + p*N_L. Outputs are
  * stacked by profile: indices [n_profiles][n_units][B]; order and margins likewise
  * (either may be NULL). ws is a separate scratch buffer (256-byte aligned) of
- * kv_evict_select_profiles_workspace bytes, not the plan's workspace. One launch
+ * kv_evict_select_profiles_workspace bytes, not the plan's workspace; its first word
+ * is this call's error word (cleared by the call, read by kv_evict_status(plan, ws,
+ * stream)). One launch
  * carries 6144 / (2 N_L) profiles (96 for N_L = 32); more go to further launches on
  * stream. Returns KVE_EINVAL for n_profiles < 1 or a non-finite coefficient, before
  * any launch. */
@@ -170,8 +172,8 @@ kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles,
                                     int32_t* order, float* margins, void* ws,
                                     void* stream);
 
-/* *bytes = scratch of kv_evict_select_profiles for n_profiles profiles (4 bytes per
- * prefix token per unit per profile). */
+/* *bytes = scratch of kv_evict_select_profiles for n_profiles profiles: a 256-byte
+ * header holding the error word, then 4 bytes per prefix token per unit per profile. */
 kve_status kv_evict_select_profiles_workspace(const kve_plan* plan,
                                               int32_t n_profiles, size_t* bytes);
 
@@ -183,8 +185,12 @@ kve_status kv_evict_select_profiles_workspace(const kve_plan* plan,
  * with the same arguments except ws; its scratch (4 bytes per prefix token per
  * unit) is a 16 MiB array compiled into the library, which every GPU that loads
  * the library keeps reserved until the process exits. It allocates nothing.
- *  * Returns KVE_EINVAL when N_L * Hkv * SL exceeds 4194304 (16 MiB / 4 B), e.g.
- *    a 32-layer, 8-KV-head request of more than 16384 tokens.
+ *  * Returns KVE_EINVAL when N_L * U * SL exceeds 4194304 (16 MiB / 4 B), where U
+ *    is the number of units per layer: Hkv, or Hq for a KVE_PLAN_PER_QUERY_HEAD
+ *    plan. E.g. a 32-layer, 8-KV-head request of more than 16384 tokens, or a
+ *    per-query-head plan with 32 layers and 32 query heads beyond 4096 tokens.
+ *  * Device-side check failures go to an error word that the library keeps beside
+ *    the array: kv_evict_status(plan, NULL, stream) reads and clears it.
  *  * The first call on a device looks up the array's device address on that
  *    device (cudaGetSymbolAddress); make that first call before any stream
  *    capture on the device.
@@ -210,10 +216,14 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k,
                            const uint16_t* v, const int32_t* indices,
                            uint16_t* k_out, uint16_t* v_out, void* stream);
 
-/* Synchronise the stream, read the device error word of ws and clear it.
+/* Synchronise the stream, read the device error word of ws and clear it. ws is the
+ * plan's workspace, the scratch of kv_evict_select_profiles, or NULL for the error
+ * word of kv_evict_select_noalloc on the current device.
  * Returns KVE_OK, KVE_ETIMEOUT (a bounded wait ran out) or KVE_ECUDA (a CUDA call
- * failed, or a device-side consistency check of kv_evict_select failed: a pool
- * position outside the unit, whose key row is then not read). */
+ * failed, or a device-side consistency check of the selection failed: a candidate
+ * pool that did not hold exactly C positions -- that unit then reports no
+ * selection, indices -1 -- or a pool position outside the unit, whose key row is
+ * then not read). */
 kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream);
 
 /* Depth profile of Eq. 6 on the host: kind 0 Global (lambda = sinh(c[0]) on every

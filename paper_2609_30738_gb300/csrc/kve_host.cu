@@ -253,13 +253,11 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
 
 }  // extern "C"
 
-namespace {
+namespace kve {
 
-// The select kernel's parameters common to every entry point; lambda1 / lambda2
-// (HOST [N_L]) may be NULL when a profile table supplies the coefficients.
 kve_status select_params(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
                          const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
-                         float* margins, kve::SelectParams* p) {
+                         float* margins, SelectParams* p) {
   const kve::Geometry& g = plan->geo;
   std::memset(p, 0, sizeof(*p));
   p->g = g;
@@ -281,6 +279,15 @@ kve_status select_params(const kve_plan* plan, const float* mu, const float* sig
   p->margins = margins;
   return KVE_OK;
 }
+
+}  // namespace kve
+
+namespace {
+
+using kve::select_params;
+
+// Bytes in front of the multi-profile scratch that hold its error word.
+constexpr size_t kProfileHeader = 256;
 
 // Scratch words of one profile (the ordered base score of every prefix token of
 // every unit), padded to 256 bytes.
@@ -319,7 +326,8 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
 
 kve_status kv_evict_select_profiles_workspace(const kve_plan* plan, int32_t n_profiles, size_t* bytes) {
   if (!plan || !bytes || n_profiles < 1 || plan->select_all) return KVE_EINVAL;
-  *bytes = static_cast<size_t>(n_profiles) * static_cast<size_t>(profile_keys_words(plan)) * sizeof(uint32_t);
+  *bytes = kProfileHeader +
+           static_cast<size_t>(n_profiles) * static_cast<size_t>(profile_keys_words(plan)) * sizeof(uint32_t);
   return KVE_OK;
 }
 
@@ -337,7 +345,12 @@ kve_status kv_evict_select_profiles(const kve_plan* plan, int32_t n_profiles, co
   kve::SelectParams p;
   const kve_status s = select_params(plan, mu, sigma, k, nullptr, nullptr, indices, order, margins, &p);
   if (s != KVE_OK) return s;
-  p.keys = static_cast<uint32_t*>(ws);
+  // the error word (cleared here, read by kv_evict_status on this ws), then the
+  // profiles' base-score keys
+  if (cudaMemsetAsync(ws, 0, sizeof(uint32_t), static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return KVE_ECUDA;
+  p.err = static_cast<uint32_t*>(ws);
+  p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + kProfileHeader);
   // the table rides in the kernel parameters; profiles beyond its capacity go to
   // further launches on the same stream
   static thread_local kve::ProfileTable table;
@@ -387,9 +400,14 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16
 }
 
 kve_status kv_evict_status(const kve_plan* plan, void* ws, void* stream) {
-  if (!plan || !ws) return KVE_EINVAL;
+  if (!plan) return KVE_EINVAL;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(st) != cudaSuccess) return KVE_ECUDA;
+  if (!ws) {
+    // the error word of the selection without a workspace, on the current device
+    ws = kve::noalloc_error_word();
+    if (!ws) return KVE_ECUDA;
+  }
   uint32_t err = 0;
   if (cudaMemcpy(&err, ws, sizeof(err), cudaMemcpyDeviceToHost) != cudaSuccess) return KVE_ECUDA;
   if (err != 0) {

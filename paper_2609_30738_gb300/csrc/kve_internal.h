@@ -134,7 +134,8 @@ struct SelectParams {
   int32_t* order;
   float* margins;
   uint32_t* keys;            // workspace scratch
-  uint32_t* err;             // workspace error word (or null): bit 2 = a pool position out of range
+  uint32_t* err;             // error word read by kv_evict_status: kErrCheck = the pool did not
+                             // hold exactly C positions, or a pool position outside the unit
   float* corr;               // workspace scratch of the every-candidate selector (or null):
                              // float2 (corr, 1/|k|) per prefix token of every unit
   float lambda1[kMaxLayers];
@@ -189,4 +190,15 @@ cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaS
 cudaError_t launch_select_profiles(const kve_plan& plan, const SelectParams& p, const ProfileTable& table,
                                    int profiles, cudaStream_t stream);
 cudaError_t launch_gather(const kve_plan& plan, const GatherParams& p, cudaStream_t stream);
+
+// The select kernel's parameters common to every selection entry point (host code,
+// kve_host.cu); lambda1 / lambda2 (HOST [N_L]) may be NULL when a profile table
+// supplies the coefficients. Leaves keys, err and corr null.
+kve_status select_params(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
+                         const float* lambda1, const float* lambda2, int32_t* indices, int32_t* order,
+                         float* margins, SelectParams* p);
+
+// Device address, on the current device, of the error word of the selection that
+// runs without a workspace (kve_select.cu); null when it cannot be looked up.
+uint32_t* noalloc_error_word();
 }  // namespace kve

@@ -476,6 +476,20 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   __syncthreads();
   const uint32_t n_above = sh.cnt;
   const uint32_t n_eq = sh.teq;
+  // Every path above leaves n_above = #{key > T} and n_eq = #{key == T} with
+  // n_above + needT = C and needT <= n_eq, so that the ties below fill the pool to
+  // exactly C positions. Should that ever fail, the pool would hold unwritten slots:
+  // the unit is then reported through the error word and gets no selection.
+  if (n_above + needT != static_cast<uint32_t>(C) || needT > n_eq || needT == 0u) {
+    if (tid == 0 && P.err) atomicOr(P.err, kErrCheck);
+    int32_t* out = P.indices + out_off + u.unit * B;
+    for (int r = tid; r < B; r += NT) out[r] = -1;
+    if (P.order)
+      for (int r = tid; r < B; r += NT) P.order[out_off + u.unit * B + r] = -1;
+    if (P.margins)
+      for (int r = tid; r < B; r += NT) P.margins[out_off + u.unit * B + r] = 0.f;
+    return;
+  }
   if (n_eq <= kTieCap) {
     // the needT lowest positions among the ties, by rank
     for (uint32_t e = tid; e < n_eq; e += NT) {
@@ -730,26 +744,42 @@ constexpr size_t kNoAllocScratchWords = size_t(4) << 20;   // 16 MiB of uint32 k
 
 // Reserved on every GPU that loads the library, for the life of the process.
 static __device__ __align__(256) uint32_t g_select_scratch[kNoAllocScratchWords];
+// Its error word (the workspace's first word plays this part for the other entry
+// points); zero at load, read and cleared by kv_evict_status with ws = NULL.
+static __device__ __align__(256) uint32_t g_noalloc_err;
 
 constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 uint32_t* g_scratch_ptr[kMaxDevices] = {};
+uint32_t* g_err_ptr[kMaxDevices] = {};
 
-// Device address of g_select_scratch on the current device (looked up once per
-// device; in host code the symbol itself is only a host-side stand-in).
-uint32_t* scratch_on_current_device() {
+// Device addresses of g_select_scratch and g_noalloc_err on the current device
+// (looked up once per device; in host code the symbols themselves are only host-side
+// stand-ins). False when the lookup fails.
+bool noalloc_addresses(uint32_t** scratch, uint32_t** err) {
   int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
   if (!g_scratch_ptr[dev]) {
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess) return nullptr;
+    void* e = nullptr;
+    if (cudaGetSymbolAddress(&p, g_select_scratch) != cudaSuccess) return false;
+    if (cudaGetSymbolAddress(&e, g_noalloc_err) != cudaSuccess) return false;
+    g_err_ptr[dev] = static_cast<uint32_t*>(e);
     g_scratch_ptr[dev] = static_cast<uint32_t*>(p);
   }
-  return g_scratch_ptr[dev];
+  *scratch = g_scratch_ptr[dev];
+  *err = g_err_ptr[dev];
+  return true;
 }
 
 }  // namespace
+
+uint32_t* noalloc_error_word() {
+  uint32_t *scratch = nullptr, *err = nullptr;
+  return noalloc_addresses(&scratch, &err) ? err : nullptr;
+}
+
 }  // namespace kve
 
 extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float* mu, const float* sigma,
@@ -760,32 +790,15 @@ extern "C" kve_status kv_evict_select_noalloc(const kve_plan* plan, const float*
   if (!plan || !mu || !sigma || !k || !lambda1 || !lambda2 || !indices || plan->select_all)
     return KVE_EINVAL;
   const Geometry& g = plan->geo;
+  // one scratch word per prefix token of every unit: N_L x (units per layer) x SL
   const size_t words = static_cast<size_t>(g.num_layers) * g.uheads * static_cast<size_t>(g.total_tokens);
   if (words > kNoAllocScratchWords) return KVE_EINVAL;   // beyond the fixed scratch
   if (((reinterpret_cast<uintptr_t>(k) | reinterpret_cast<uintptr_t>(mu) |
         reinterpret_cast<uintptr_t>(sigma)) & 15u) != 0)
     return KVE_EINVAL;   // the header asks every pointer to be 16-byte aligned
-  uint32_t* scratch = scratch_on_current_device();
-  if (!scratch) return KVE_ECUDA;
   SelectParams p;
-  memset(&p, 0, sizeof(p));
-  p.g = g;
-  p.budget = plan->cfg.budget;
-  p.pool_kernel = plan->cfg.pool_kernel;
-  p.cand_factor = plan->cfg.candidate_factor;
-  p.norm_eps = plan->cfg.norm_eps;
-  for (int l = 0; l < g.num_layers; ++l) {
-    if (!isfinite(lambda1[l]) || !isfinite(lambda2[l])) return KVE_EINVAL;
-    p.lambda1[l] = lambda1[l];
-    p.lambda2[l] = lambda2[l];
-    p.layer_budget[l] = plan->layer_budget[l];
-  }
-  p.mu = mu;
-  p.sigma = sigma;
-  p.k = k;
-  p.indices = indices;
-  p.order = order;
-  p.margins = margins;
-  p.keys = scratch;
+  const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
+  if (s != KVE_OK) return s;
+  if (!noalloc_addresses(&p.keys, &p.err)) return KVE_ECUDA;
   return launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
 }

@@ -191,7 +191,8 @@ class Plan:
                        stream=None):
         """kv_evict_select without a workspace, for callers that cannot allocate
         device memory while they evict; its scratch is a fixed 16 MiB array inside
-        the library (at most N_L * Hkv * SL = 4194304 tokens per call)."""
+        the library (at most N_L * units per layer * SL = 4194304 tokens per call).
+        status(None) reads its error word."""
         l1 = np.ascontiguousarray(lambda1, dtype=np.float32)
         l2 = np.ascontiguousarray(lambda2, dtype=np.float32)
         assert l1.shape == (self.spec["num_layers"],) and l2.shape == l1.shape
@@ -233,7 +234,8 @@ class Plan:
                                       _ptr(v_out), _stream_ptr(stream)), "kv_evict_gather")
 
     def status(self, ws, stream=None) -> int:
-        """Synchronise, return the device status (KVE_OK or KVE_ETIMEOUT) and clear it."""
+        """Synchronise, return the device status (KVE_OK, KVE_ETIMEOUT or KVE_ECUDA) of
+        ws and clear it; ws = None reads the error word of select_noalloc."""
         return int(_lib().kv_evict_status(self._h, _ptr(ws), _stream_ptr(stream)))
 
 

@@ -88,9 +88,12 @@ def unit_tensors(seed, r, layer, L, Hkv, G, W, d=128, salient_frac=0.0, noise=0.
     return k, v, q
 
 
-def make_batch(spec: dict, seed: int = 2609, device="cpu", with_values: bool = True):
+def make_batch(spec: dict, seed: int = 2609, device="cpu", with_values: bool = True,
+               request_ids=None):
     """Inputs of a whole call in the library's layouts (see include/kv_evict.h):
-    q_win [N_L][n_req][Hq][W][d], k/v [N_L][Hkv][SL][d], all bf16 (torch tensors)."""
+    q_win [N_L][n_req][Hq][W][d], k/v [N_L][Hkv][SL][d], all bf16 (torch tensors).
+    request_ids[j] (default j) is the request number that seeds the j-th request, so
+    that a subset of a batch's requests gets the same tensors as in the whole batch."""
     N_L, Hq, Hkv, d, W = (spec["num_layers"], spec["num_q_heads"], spec["num_kv_heads"],
                           spec["head_dim"], spec["window"])
     lens = [int(x) for x in spec["seq_lens"]]
@@ -99,10 +102,12 @@ def make_batch(spec: dict, seed: int = 2609, device="cpu", with_values: bool = T
     q_win = torch.empty((N_L, len(lens), Hq, W, d), dtype=torch.bfloat16, device=device)
     k = torch.empty((N_L, Hkv, SL, d), dtype=torch.bfloat16, device=device)
     v = torch.empty((N_L, Hkv, SL, d), dtype=torch.bfloat16, device=device) if with_values else None
+    ids = list(range(len(lens))) if request_ids is None else [int(x) for x in request_ids]
+    assert len(ids) == len(lens)
     off = 0
     for r, L in enumerate(lens):
         for layer in range(N_L):
-            kk, vv, qq = unit_tensors(seed, r, layer, L, Hkv, G, W, d,
+            kk, vv, qq = unit_tensors(seed, ids[r], layer, L, Hkv, G, W, d,
                                       salient_frac=spec.get("salient_frac", 0.0), device=device)
             k[layer, :, off:off + L] = kk.to(torch.bfloat16)
             if with_values:

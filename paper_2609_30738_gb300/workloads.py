@@ -73,3 +73,32 @@ def lambda_arrays(spec: dict, profile_fn):
         return (np.full(N_L, float(l1)),
                 -0.6 + 1.2 * ((ell - mid) / mid) ** 2 - 0.6)
     raise ValueError(kind)
+
+
+def partition_requests(seq_lens, world: int):
+    """Split the requests of one batch across `world` ranks, balanced by prefix tokens
+    (the score kernel's work is proportional to them): longest first, each to the
+    rank with the fewest tokens so far (ties to the lower rank). Returns one sorted
+    list of request indices per rank; every request goes to exactly one rank. A
+    rank may get none when there are fewer requests than ranks."""
+    loads = [0] * world
+    parts = [[] for _ in range(world)]
+    for r in sorted(range(len(seq_lens)), key=lambda i: (-int(seq_lens[i]), i)):
+        j = min(range(world), key=lambda w: (loads[w], w))
+        parts[j].append(r)
+        loads[j] += int(seq_lens[r])
+    return [sorted(p) for p in parts]
+
+
+def request_layout(seq_lens, num_layers: int, unit_heads: int):
+    """Per request r, (first unit, units, first mu/sigma element, elements) in the
+    layouts of include/kv_evict.h: units are request-major (N_L * unit_heads per
+    request) and mu / sigma are packed per request (N_L * unit_heads * L_r)."""
+    out = []
+    unit = elem = 0
+    for L in seq_lens:
+        n_u = num_layers * unit_heads
+        out.append((unit, n_u, elem, n_u * int(L)))
+        unit += n_u
+        elem += n_u * int(L)
+    return out

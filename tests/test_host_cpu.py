@@ -140,7 +140,7 @@ def test_select_profiles_validation_without_gpu():
     words = 3 * 8 * (2048 + 777)
     padded = (words + 63) // 64 * 64
     for n in (1, 2, 14):
-        assert p.select_profiles_workspace(n) == n * padded * 4
+        assert p.select_profiles_workspace(n) == 256 + n * padded * 4   # error-word header
     with pytest.raises(K.KvEvictError) as e:
         p.select_profiles_workspace(0)
     assert e.value.status == K.KVE_EINVAL
@@ -220,3 +220,27 @@ def test_gather_refuses_pageable_host_memory_without_gpu():
     buf = np.zeros(1 << 16, dtype=np.uint8)
     ptr = buf.ctypes.data + (-buf.ctypes.data) % 16            # 16-byte aligned
     assert K.library().kv_evict_gather(p._h, ptr, ptr, ptr, ptr, ptr, None) == K.KVE_EINVAL
+
+
+def test_noalloc_size_limit_counts_units_per_layer_without_gpu():
+    """kv_evict_select_noalloc refuses, before any CUDA call, a plan whose scratch
+    (one word per prefix token of every unit) exceeds its fixed 4194304-word array;
+    a per-query-head plan has Hq units per layer, not Hkv, so it reaches the limit
+    G times sooner."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    lib = K.library()
+    lam = np.zeros(32, np.float32)
+    fake = ctypes.c_void_p(1 << 20)
+    spec = _spec(num_layers=32)
+    # 32 layers x 32 query heads x 4100 tokens = 4198400 words: over the limit
+    perq = K.Plan(spec, [4100], per_query_head=True)
+    assert perq.score_elems > 4194304
+    assert lib.kv_evict_select_noalloc(perq._h, fake, fake, fake, lam.ctypes.data, lam.ctypes.data,
+                                       fake, None, None, None) == K.KVE_EINVAL
+    # the same prefix grouped per KV head needs 1049600 words: within the limit
+    assert K.Plan(spec, [4100]).score_elems <= 4194304
+    # 32 layers x 8 KV heads x 16385 tokens: over the limit
+    big = K.Plan(spec, [16385])
+    assert lib.kv_evict_select_noalloc(big._h, fake, fake, fake, lam.ctypes.data, lam.ctypes.data,
+                                       fake, None, None, None) == K.KVE_EINVAL

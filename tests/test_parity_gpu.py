@@ -344,12 +344,15 @@ def test_near_constant_columns_two_pass(window, L):
 
 
 @pytest.mark.parametrize("L,B,lams", [(1500, 32, (0.5, -0.5)), (5000, 24, (0.3, 0.6)),
-                                      (2600, 40, (0.0, 0.0)), (700, 8, (-0.3, -3.0))])
+                                      (2600, 40, (0.0, 0.0)), (700, 8, (-0.3, -3.0)),
+                                      (4096, 160, (0.5, -0.5)), (3000, 100, (0.3, -0.8))])
 def test_every_candidate_greedy(L, B, lams):
     """candidate_factor = 0 beyond the 512-slot pool (the unrestricted ablation of
     Section 3.2): the every-candidate selector -- bounds brought up to date on demand
     for lambda2 <= 0, every value after each admission for lambda2 > 0 -- against the
-    oracle's full greedy over all Lc candidates, margins included."""
+    oracle's full greedy over all Lc candidates, margins included. B = 160 and 100
+    run past the 96 admitted keys the selector stages in shared memory (the later
+    ones are read from K) and B = 100 ends in a partial group of 16 admissions."""
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[L], budget=B, candidate_factor=0,
                   lambdas=("global",) + lams)
     batch = synth.make_batch(spec, seed=L + B)
@@ -422,7 +425,7 @@ def test_bounded_wait_reports_timeout_and_gpu_stays_usable():
     PT.check_mu_sigma(bufs.mu[:1024].cpu().numpy(), bufs.sigma[:1024].cpu().numpy(), mu_ref, sg_ref)
 
 
-# ---------------------------------------------------------------- full-size workloads, sampled units
+# ---------------------------------------------------------------- full-size workloads, every unit
 
 
 FULL = ["mistral-32layer-L8192", "mistral-32layer-L32768-B32", "mistral-32layer-L32768-B64",
@@ -430,31 +433,39 @@ FULL = ["mistral-32layer-L8192", "mistral-32layer-L32768-B32", "mistral-32layer-
 
 
 @pytest.mark.parametrize("name", FULL)
-def test_full_size_sampled_units(name):
+def test_full_size_every_unit(name):
+    """Each full-size workload in the launch configuration bench.py times: every
+    unit's mu and sigma against the oracle's Eq. 1 / Eq. 3 and its admissions
+    replayed through the oracle's selection (spawned workers on the host cores),
+    every unit's compact cache against plain indexing, and a few units' gathers
+    against the oracle. The error statistics are printed, and appended as one JSON
+    line to the file named by KVE_PARITY_REPORT when that is set."""
+    import json
+    import os
+    import time
+    from tests import fullsize
     spec = WORKLOADS[name]
     batch = synth.make_batch(spec, seed=2609, device=DEV)
     plan, bufs, _, lam = _run(spec, batch)
     seq = batch["seq_lens"]
     N_L, Hkv = spec["num_layers"], spec["num_kv_heads"]
-    # properties on every unit: each unit's mu sums to 1 (every row is a distribution)
-    sums = []
-    off = 0
-    for r, L in enumerate(seq):
-        seg = bufs.mu[N_L * Hkv * off: N_L * Hkv * (off + L)].view(N_L * Hkv, L).double().sum(1)
-        sums.append(seg)
-        off += L
-    sums = torch.cat(sums)
-    assert torch.all((sums - 1).abs() < 1e-3), float((sums - 1).abs().max())
-    idx = bufs.indices
-    B = spec["budget"]
-    assert torch.all(idx[:, 1:] > idx[:, :-1]), "indices ascending and unique"
-    # oracle on sampled units: first, last, middle layer; shortest and longest request
-    r_lo = int(np.argmin(seq))
-    r_hi = int(np.argmax(seq))
-    units = sorted({(0, 0, 0), (r_hi, N_L - 1, Hkv - 1), (r_lo, N_L // 2, 3), (r_hi, 11, 5),
-                    (len(seq) - 1, 21, 2)})
-    worst, swaps = _check_units(spec, batch, plan, bufs, lam, units)
-    print(f"{name}: max mu rel err {worst:.2e}, near-tie swaps {swaps}")
+    t0 = time.time()
+    stats = fullsize.check_every_unit(spec, batch, plan, bufs, lam)
+    assert stats["units"] == len(seq) * N_L * Hkv
+    assert not stats["failures"], stats["failures"][:5]
+    fullsize.check_every_gather(spec, batch, plan, bufs)
+    r_lo, r_hi = int(np.argmin(seq)), int(np.argmax(seq))
+    units = sorted({(0, 0, 0), (r_hi, N_L - 1, Hkv - 1), (r_lo, N_L // 2, 3)})
+    _check_units(spec, batch, plan, bufs, lam, units)
+    line = dict(workload=name, units=stats["units"], mu_rel_max=stats["mu_rel"],
+                sigma_rel_max=stats["sigma_rel"], sigma_checks_needing_floor=stats["sigma_floor"],
+                sigma_tol_ratio_max=stats["sigma_ratio"], swaps=stats["swaps"],
+                host_check_s=round(time.time() - t0, 1), workers=os.cpu_count())
+    print(json.dumps(line))
+    path = os.environ.get("KVE_PARITY_REPORT")
+    if path:
+        with open(path, "a") as f:
+            f.write(json.dumps(line) + "\n")
 
 
 def test_layer_chunks_with_host_values_full_size():

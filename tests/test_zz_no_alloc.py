@@ -3,10 +3,11 @@
 Serving engines that reserve almost all of HBM for their own KV-cache pool, and
 plugin hosts that hand a kernel only its inputs and outputs, cannot give the
 selector a workspace. This entry point keeps the selector's scratch in a fixed
-array inside the library instead. These tests check, through the C ABI, that two
-calls in a row return what the workspace entry point returns for the same inputs,
-and that a request too large for the fixed array is refused before any launch.
-The file is named so that pytest collects it last.
+array inside the library instead, and its device-side error word beside it. These
+tests check, through the C ABI, that two calls in a row return what the workspace
+entry point returns for the same inputs, that the library's error word reads clean
+after them, and that requests too large for the fixed array are refused before any
+launch. The file is named so that pytest collects it last.
 """
 
 import numpy as np
@@ -34,12 +35,14 @@ def _select_both(K, plan, bufs, k, lam1, lam2):
     """Workspace entry point, then the no-allocation one, on the same mu/sigma."""
     n, B = bufs.indices.shape
     plan.select(bufs.mu, bufs.sigma, k, lam1, lam2, bufs.indices, bufs.ws, bufs.order, bufs.margins)
+    assert plan.status(bufs.ws) == K.KVE_OK
     ref = (bufs.indices.clone(), bufs.order.clone(), bufs.margins.clone())
     idx = torch.full((n, B), -7, dtype=torch.int32, device=k.device)
     order = torch.full((n, B), -7, dtype=torch.int32, device=k.device)
     margins = torch.full((n, B), float("nan"), dtype=torch.float32, device=k.device)
     plan.select_noalloc(bufs.mu, bufs.sigma, k, lam1, lam2, idx, order, margins)
-    assert plan.status(bufs.ws) == K.KVE_OK
+    # the no-allocation call's own error word (kept in the library, not in bufs.ws)
+    assert plan.status(None) == K.KVE_OK
     return ref, (idx, order, margins)
 
 
@@ -72,11 +75,17 @@ def test_noalloc_matches_workspace_select_twice(K):
 
 
 def test_noalloc_refuses_requests_beyond_its_array(K):
+    lib = K.library()
+    lam = np.zeros(32, np.float32)
     # 32 layers x 8 KV heads x 20000 tokens = 5.12 M scores > 4194304 (16 MiB)
     spec = scaled(WORKLOADS["mistral-32layer-L8192"], seq_lens=[20000])
     plan = K.Plan(spec, spec["seq_lens"])
-    lib = K.library()
-    lam = np.zeros(32, np.float32)
     st = lib.kv_evict_select_noalloc(plan._h, 16, 16, 16, lam.ctypes.data, lam.ctypes.data, 16,
                                      None, None, None)
     assert st == K.KVE_EINVAL
+    # a per-query-head plan counts Hq units per layer: 32 x 32 x 4100 > 4194304
+    perq = K.Plan(scaled(spec, seq_lens=[4100]), [4100], per_query_head=True)
+    st = lib.kv_evict_select_noalloc(perq._h, 16, 16, 16, lam.ctypes.data, lam.ctypes.data, 16,
+                                     None, None, None)
+    assert st == K.KVE_EINVAL
+    assert perq.status(None) == K.KVE_OK
