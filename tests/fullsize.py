@@ -10,11 +10,13 @@ statistics and replays the GPU's admission order through the oracle's selection
 (tests/parity.py: tolerances, near-tie swaps) and returns error statistics:
 
   mu_rel        max |mu - mu_ref| / mu_ref
-  sigma_rel     max |sigma - sigma_ref| / sigma_ref (no floor)
-  sigma_floor   checks whose |sigma - sigma_ref| exceeds 1e-3 sigma_ref, i.e. that
-                pass only through the mu-proportional floor of the sigma tolerance
-  sigma_ratio   max |sigma - sigma_ref| / tolerance (<= 1 passes)
-  swaps         accepted near-tie swaps (unit, step, gpu pick, oracle pick, gap)
+  sigma_rel     max |sigma - sigma_ref| / sigma_ref over sigma_ref >= 1e-20
+  sigma_tiny    keys with 0 < sigma_ref < 1e-20 (A below about 2^-103: the kernel's
+                fp32 squares underflow there, and the 1e-30 absolute floor holds)
+  sigma_floor   checks whose |sigma - sigma_ref| exceeds 1e-3 sigma_ref + 1e-30,
+                i.e. that would need a mu-proportional floor (none is applied here)
+  sigma_ratio   max |sigma - sigma_ref| / (1e-3 sigma_ref + 1e-4 mu_ref + 1e-30)
+  swaps         accepted near-tie swaps (unit, step, gpu pick, oracle pick, gap, kind)
   failures      messages of every check that failed
 """
 
@@ -32,8 +34,8 @@ def _slice_check(task):
     from tests import parity as PT
     (r, layer, L, W, G, B, lam1, lam2, pool_kernel, cand_factor, eps,
      q_bits, k_bits, mu, sigma, order, indices, margins) = task
-    out = dict(units=0, mu_rel=0.0, sigma_rel=0.0, sigma_floor=0, sigma_ratio=0.0, swaps=[],
-               failures=[])
+    out = dict(units=0, mu_rel=0.0, sigma_rel=0.0, sigma_tiny=0, sigma_floor=0, sigma_ratio=0.0,
+               swaps=[], failures=[])
     for h in range(k_bits.shape[0]):
         tag = f"unit(r={r},l={layer},h={h})"
         qf = O.bf16_bits_to_f64(q_bits[h])
@@ -43,9 +45,10 @@ def _slice_check(task):
         dmu = np.abs(m - mu_ref)
         dsg = np.abs(s - sg_ref)
         out["mu_rel"] = max(out["mu_rel"], float((dmu / np.maximum(mu_ref, 1e-300)).max()))
-        pos = sg_ref > 0
+        pos = sg_ref >= 1e-20
         if pos.any():
             out["sigma_rel"] = max(out["sigma_rel"], float((dsg[pos] / sg_ref[pos]).max()))
+        out["sigma_tiny"] += int(np.count_nonzero((sg_ref > 0) & (sg_ref < 1e-20)))
         out["sigma_floor"] += int(np.count_nonzero(dsg > PT.SIGMA_RTOL * sg_ref + PT.ABS_FLOOR))
         tol = PT.SIGMA_RTOL * sg_ref + PT.SIGMA_MU_FLOOR * mu_ref + PT.ABS_FLOOR
         out["sigma_ratio"] = max(out["sigma_ratio"], float((dsg / tol).max()))
@@ -93,12 +96,13 @@ def check_every_unit(spec, batch, plan, bufs, lambdas, workers=None):
     workers = workers or max(1, os.cpu_count() or 1)
     for var in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         os.environ[var] = "1"
-    total = dict(units=0, mu_rel=0.0, sigma_rel=0.0, sigma_floor=0, sigma_ratio=0.0, swaps=[],
-                 failures=[])
+    total = dict(units=0, mu_rel=0.0, sigma_rel=0.0, sigma_tiny=0, sigma_floor=0, sigma_ratio=0.0,
+                 swaps=[], failures=[])
 
     def merge(res):
         total["units"] += res["units"]
         total["sigma_floor"] += res["sigma_floor"]
+        total["sigma_tiny"] += res["sigma_tiny"]
         for key in ("mu_rel", "sigma_rel", "sigma_ratio"):
             total[key] = max(total[key], res[key])
         total["swaps"] += res["swaps"]

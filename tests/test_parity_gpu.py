@@ -46,7 +46,7 @@ def _mu_offset(spec, seq_lens, r, layer, h):
     return N_L * Hkv * sum(seq_lens[:r]) + (layer * Hkv + h) * seq_lens[r]
 
 
-def _check_units(spec, batch, plan, bufs, lambdas, units, sel_mode="replay"):
+def _check_units(spec, batch, plan, bufs, lambdas, units, sigma_mu_floor=0.0):
     """Oracle comparison of the listed units (r, layer, h). Returns max mu rel error
     and the list of near-tie swaps."""
     seq = batch["seq_lens"]
@@ -67,7 +67,8 @@ def _check_units(spec, batch, plan, bufs, lambdas, units, sel_mode="replay"):
         mu_ref, sg_ref = O.score_unit(qf, kf, L, W, G)
         o = _mu_offset(spec, seq, r, layer, h)
         tag = f"unit(r={r},l={layer},h={h})"
-        worst = max(worst, PT.check_mu_sigma(mu_all[o:o + L], sg_all[o:o + L], mu_ref, sg_ref, tag))
+        worst = max(worst, PT.check_mu_sigma(mu_all[o:o + L], sg_all[o:o + L], mu_ref, sg_ref, tag,
+                                             sigma_mu_floor=sigma_mu_floor))
         ui = _unit_index(spec, seq, r, layer, h)
         Bl = plan.layer_budgets[layer]
         swaps += PT.check_selection(ord_all[ui], idx_all[ui], mu_ref, sg_ref, kf, L, W, Bl,
@@ -340,7 +341,8 @@ def test_near_constant_columns_two_pass(window, L):
     batch = synth.make_batch(spec, seed=31)
     batch["q_win"] = torch.zeros_like(batch["q_win"])
     plan, bufs, _, lam = _run(spec, batch)
-    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
+    _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]),
+                 sigma_mu_floor=PT.SIGMA_MU_FLOOR)
 
 
 @pytest.mark.parametrize("L,B,lams", [(1500, 32, (0.5, -0.5)), (5000, 24, (0.3, 0.6)),
@@ -458,7 +460,8 @@ def test_full_size_every_unit(name):
     units = sorted({(0, 0, 0), (r_hi, N_L - 1, Hkv - 1), (r_lo, N_L // 2, 3)})
     _check_units(spec, batch, plan, bufs, lam, units)
     line = dict(workload=name, units=stats["units"], mu_rel_max=stats["mu_rel"],
-                sigma_rel_max=stats["sigma_rel"], sigma_checks_needing_floor=stats["sigma_floor"],
+                sigma_rel_max=stats["sigma_rel"], sigma_tiny=stats["sigma_tiny"],
+                sigma_checks_needing_floor=stats["sigma_floor"],
                 sigma_tol_ratio_max=stats["sigma_ratio"], swaps=stats["swaps"],
                 host_check_s=round(time.time() - t0, 1), workers=os.cpu_count())
     print(json.dumps(line))
