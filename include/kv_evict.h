@@ -23,13 +23,18 @@
  *  * The window rows of unit (r, l, h) are the G query heads h*G .. h*G+G-1, each
  *    with its W window queries: n = G*W rows, row index g*W + w, at token position
  *    L_r - W + w. Causal masking: that row attends to keys 0 .. L_r - W + w.
- *  * All tensors are dense, row-major, in device memory, allocated and owned by
- *    the caller. bf16 tensors are passed as uint16_t bit patterns.
+ *  * All tensors are row-major, in device memory, allocated and owned by the
+ *    caller; all but k and v are dense. bf16 tensors are passed as uint16_t bit
+ *    patterns.
  *      q_win  [N_L][n_req][Hq][W][d]      bf16  window queries (after RoPE)
  *      k, v   [N_L][Hkv][SL][d]           bf16  prefix keys/values (after RoPE);
  *                                               request r occupies tokens
  *                                               off_r .. off_r + L_r - 1,
- *                                               off_r = L_0 + ... + L_{r-1}
+ *                                               off_r = L_0 + ... + L_{r-1}.
+ *                                               Dense by default; any other
+ *                                               strides between layers, heads and
+ *                                               tokens through
+ *                                               kv_evict_plan_set_kv_strides
  *      mu, sigma  packed per request: request r holds [N_L][Hkv][L_r] fp32 at
  *                 element offset N_L*Hkv*off_r
  *      indices    [n_req][N_L][Hkv][B] int32, kept candidate positions in
@@ -123,6 +128,19 @@ kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens,
                             size_t* workspace_bytes);
 
 void kv_evict_plan_destroy(kve_plan* plan);
+
+/* Layout of k and v for later calls with this plan, so that a serving engine's cache
+ * is read in place: strides[3] = element strides between layers, KV heads and
+ * tokens (in that order) of the prefix keys (k_strides) and values (v_strides);
+ * element (layer l, KV head h, token t, dim j) sits at l*s[0] + h*s[1] + t*s[2] + j,
+ * with t = off_r + i for key i of request r (off_r as above). A row of d elements
+ * stays contiguous. NULL is the dense default {Hkv*SL*d, SL*d, d}; a token-major
+ * cache [N_L][SL][Hkv][d] is {SL*Hkv*d, d, Hkv*d}. Every stride must be a multiple
+ * of 8 elements (16 bytes) and below 2^37, and the token stride at least d;
+ * otherwise KVE_EINVAL and the plan is unchanged. Call it before the plan is used
+ * on any stream; it changes the plan (not thread-safe with calls that use it). */
+kve_status kv_evict_plan_set_kv_strides(kve_plan* plan, const int64_t* k_strides,
+                                        const int64_t* v_strides);
 
 /* Test hook: limit (ns) of every device-side bounded wait of later calls with this
  * plan (default 2e9), and a fault to inject on the host-chosen unit 0:

@@ -54,6 +54,22 @@ bool encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// k viewed as a 4-D tensor (d, token, KV head, layer) with the plan's element strides;
+// boxes of 64 elements x 128 tokens with the 128-byte swizzle, tokens past SL read as zero.
+bool encode_keys(CUtensorMap* map, const void* base, const kve::Geometry& g) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[4] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(g.total_tokens),
+                        static_cast<cuuint64_t>(g.hkv), static_cast<cuuint64_t>(g.num_layers)};
+  cuuint64_t strides[3] = {static_cast<cuuint64_t>(g.k_st) * 2, static_cast<cuuint64_t>(g.k_sh) * 2,
+                           static_cast<cuuint64_t>(g.k_sl) * 2};
+  cuuint32_t box[4] = {64, 128, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int device_sms() {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -177,19 +193,23 @@ kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens, int3
   g.req_unit_base[n_req] = units;
   g.req_item_base[n_req] = items;
   g.total_tokens = off;
+  // the dense layouts [N_L][Hkv][SL][d] until kv_evict_plan_set_kv_strides
+  g.k_st = g.v_st = kHeadDim;
+  g.k_sh = g.v_sh = off * kHeadDim;
+  g.k_sl = g.v_sl = static_cast<int64_t>(c.num_kv_heads) * off * kHeadDim;
   g.n_units = units;
   g.n_items = items;
   const int64_t max_cand = c.candidate_factor == 0 ? max_lc
                                                    : std::min<int64_t>(int64_t(c.candidate_factor) * c.budget, max_lc);
-  // TMA row coordinates are 32-bit; the select kernel holds its pool in shared memory
-  const int64_t k_rows = static_cast<int64_t>(c.num_layers) * c.num_kv_heads * off;
+  // TMA coordinates (window rows of q_win, tokens of k) are 32-bit; the select kernel
+  // holds its pool in shared memory
   const int64_t q_rows = static_cast<int64_t>(c.num_layers) * n_req * c.num_q_heads * c.window;
   // candidate_factor = 0 beyond the pooled selector's pool runs the every-candidate
   // selector (Lc <= kMaxAllCand, B <= kMaxAllBudget)
   plan->select_all = (c.candidate_factor == 0 && max_lc > kve::kMaxPoolCand) ? 1 : 0;
   const bool cand_ok = plan->select_all ? (max_lc <= kve::kMaxAllCand && c.budget <= kve::kMaxAllBudget)
                                         : max_cand <= kve::kMaxPoolCand;
-  if (!cand_ok || k_rows >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
+  if (!cand_ok || off >= (int64_t(1) << 31) - 256 || q_rows >= (int64_t(1) << 31) - 256 ||
       2 * items >= (int64_t(1) << 31) || units >= (int64_t(1) << 31)) {
     delete plan;
     return KVE_EINVAL;
@@ -211,6 +231,29 @@ kve_status kv_evict_plan_ex(const kve_config* cfg, const int64_t* seq_lens, int3
 
 void kv_evict_plan_destroy(kve_plan* plan) { delete plan; }
 
+kve_status kv_evict_plan_set_kv_strides(kve_plan* plan, const int64_t* k_strides, const int64_t* v_strides) {
+  if (!plan) return KVE_EINVAL;
+  kve::Geometry& g = plan->geo;
+  const int64_t dense[3] = {static_cast<int64_t>(g.hkv) * g.total_tokens * kHeadDim, g.total_tokens * kHeadDim,
+                            kHeadDim};
+  const int64_t* ks = k_strides ? k_strides : dense;
+  const int64_t* vs = v_strides ? v_strides : dense;
+  // each stride a multiple of 8 elements (16 bytes, the TMA and vector-load rule) and
+  // below 2^37 elements (TMA strides below 2^40 bytes); a token step of at least one row
+  for (const int64_t* st : {ks, vs}) {
+    for (int i = 0; i < 3; ++i)
+      if (st[i] < 0 || st[i] % 8 != 0 || st[i] >= (int64_t(1) << 37)) return KVE_EINVAL;
+    if (st[2] < kHeadDim) return KVE_EINVAL;
+  }
+  g.k_sl = ks[0];
+  g.k_sh = ks[1];
+  g.k_st = ks[2];
+  g.v_sl = vs[0];
+  g.v_sh = vs[1];
+  g.v_st = vs[2];
+  return KVE_OK;
+}
+
 kve_status kv_evict_plan_set_debug(kve_plan* plan, uint64_t wait_limit_ns, int32_t fault) {
   if (!plan || wait_limit_ns == 0 || fault < 0 || fault > 1) return KVE_EINVAL;
   plan->wait_limit_ns = wait_limit_ns;
@@ -228,8 +271,7 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
   if (sms <= 0) return KVE_ECUDA;
   CUtensorMap tm_q, tm_k;
   const int64_t q_rows = static_cast<int64_t>(g.num_layers) * g.n_req * g.hq * g.window;
-  const int64_t k_rows = static_cast<int64_t>(g.num_layers) * g.hkv * g.total_tokens;
-  if (!encode_rows(&tm_q, q_win, q_rows) || !encode_rows(&tm_k, k, k_rows)) return KVE_ECUDA;
+  if (!encode_rows(&tm_q, q_win, q_rows) || !encode_keys(&tm_k, k, g)) return KVE_ECUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* w = static_cast<uint8_t*>(ws);
   if (cudaMemsetAsync(w, 0, plan->ws.clear_end, st) != cudaSuccess) return KVE_ECUDA;

@@ -4,6 +4,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -31,6 +32,10 @@ struct Geometry {
                                         // when every query head selects for itself
   int32_t ugroup;                       // query heads per unit: group, or 1
   int64_t total_tokens;                 // SL
+  // element strides of k and v between layers, KV heads and tokens (a row is d
+  // contiguous elements); the dense default is token d, head SL*d, layer Hkv*SL*d
+  int64_t k_sl, k_sh, k_st;
+  int64_t v_sl, v_sh, v_st;
   int64_t n_units;                      // n_req * N_L * uheads
   int64_t n_items;                      // score work items (sum over units of splits)
   int32_t req_len[kMaxReq];             // L_r
@@ -49,7 +54,10 @@ struct UnitInfo {
   int32_t splits;      // items of this unit
   int64_t local;       // unit index within its request
   int64_t q_row0;      // first window row in q_win viewed as [rows][d]
-  int64_t k_row0;      // first key row in k viewed as [rows][d]
+  int32_t kvh;         // the KV head whose keys the unit reads
+  int64_t tok0;        // token index of the unit's first key in k / v (off_r)
+  int64_t k_off;       // element offset of the unit's first key row in k: key i at k_off + i * k_st
+  int64_t v_off;       // the same in v
   int64_t mu_off;      // first element of this unit in mu / sigma
   int64_t item0;       // first score item of this unit
 };
@@ -70,7 +78,10 @@ __host__ __device__ inline UnitInfo unit_info(const Geometry& g, int64_t unit) {
   u.q_row0 = ((static_cast<int64_t>(u.layer) * g.n_req + r) * g.hq +
               static_cast<int64_t>(u.h) * g.ugroup) * g.window;
   const int kvh = g.ugroup == g.group ? u.h : u.h / g.group;   // the KV head the unit reads
-  u.k_row0 = (static_cast<int64_t>(u.layer) * g.hkv + kvh) * g.total_tokens + g.req_tok_off[r];
+  u.kvh = kvh;
+  u.tok0 = g.req_tok_off[r];
+  u.k_off = u.layer * g.k_sl + kvh * g.k_sh + u.tok0 * g.k_st;
+  u.v_off = u.layer * g.v_sl + kvh * g.v_sh + u.tok0 * g.v_st;
   u.mu_off = static_cast<int64_t>(g.num_layers) * g.uheads * g.req_tok_off[r] + local * u.L;
   u.item0 = g.req_item_base[r] + local * u.splits;
   return u;
@@ -182,6 +193,32 @@ struct kve_plan {
 };
 
 namespace kve {
+// Programmatic dependent launch: a kernel launched with launch_after_previous may be
+// scheduled while the previous kernel on its stream finishes; it waits here, before
+// touching memory, until that kernel has completed and its writes are visible (a no-op
+// for a kernel launched without the attribute).
+__device__ __forceinline__ void wait_previous_kernel() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Launch `fn` on `stream` after the previous kernel of the stream, overlapping its
+// launch with that kernel's tail (programmatic stream serialization).
+template <class... KArgs, class... Args>
+cudaError_t launch_after_previous(void (*fn)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                  cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, fn, std::forward<Args>(args)...);
+}
+
 // Kernel launchers (defined next to their kernels).
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
                          const ScoreParams& p, int ctas, cudaStream_t stream);

@@ -79,7 +79,9 @@ struct ItemDesc {
   int32_t ntiles;
   int32_t L;         // prefix length of the unit
   int32_t splits;    // items of the unit
-  int32_t pad;
+  int32_t tok0;      // K tile coordinates: the unit's first token, KV head and layer
+  int32_t kvh;
+  int32_t layer;
 };
 
 struct Claim {
@@ -657,7 +659,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           item_range(u, split, &d.tile0, &d.ntiles);
           d.L = u.L;
           d.splits = u.splits;
-          d.pad = 0;
+          d.tok0 = static_cast<int32_t>(u.tok0);
+          d.kvh = u.kvh;
+          d.layer = u.layer;
         } else {
           d.p = -1;
         }
@@ -687,10 +691,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
           }
-          const int32_t y = static_cast<int32_t>(u.k_row0 + (tile0 + t) * kTileKeys);
+          const int32_t y = d.tok0 + (tile0 + t) * kTileKeys;
           mbar_arrive_expect_tx(&ctl.k_full[ks], kTileBytes);
-          tma_load_2d_hint(kbuf + ks * kTileBytes, &tm_k, 0, y, &ctl.k_full[ks], pol);
-          tma_load_2d_hint(kbuf + ks * kTileBytes + kHalfBytes, &tm_k, 64, y, &ctl.k_full[ks], pol);
+          tma_load_4d_hint(kbuf + ks * kTileBytes, &tm_k, 0, y, d.kvh, d.layer, &ctl.k_full[ks], pol);
+          tma_load_4d_hint(kbuf + ks * kTileBytes + kHalfBytes, &tm_k, 64, y, d.kvh, d.layer,
+                           &ctl.k_full[ks], pol);
           k_used |= 1u << ks;
           k_last = (k_last & ~(1u << ks)) | (((ki / kKStages) & 1u) << ks);
           ++ki;

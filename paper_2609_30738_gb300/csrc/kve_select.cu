@@ -8,12 +8,12 @@
 //     the top 4B tokens) by an MSB-first radix select with 12/12/8-bit digits;
 //     ties at the cut go to the lower positions;
 //  3. normalise s~ = s / max(max s, eps) (Eq. 5) and stage the candidate keys
-//     (bf16) and their inverse norms in shared memory, candidates sorted by
-//     position so that "lower slot" means "lower position";
+//     (bf16) and their inverse norms in shared memory;
 //  4. admit min(B, C) candidates greedily (Eq. 5): value s~ + lambda2 corr, ties to
-//     the lower position; after every admission j, corr_i <- max(corr_i,
-//     cos(k_i, k_j)), which is Eq. 4 for the grown set (corr starts at 0, which is
-//     both corr(i, {}) and the clamp at 0);
+//     the lower position (the argmax compares position << 9 | slot after the value);
+//     after every admission j, corr_i <- max(corr_i, cos(k_i, k_j)), which is Eq. 4
+//     for the grown set (corr starts at 0, which is both corr(i, {}) and the clamp
+//     at 0);
 //  5. write the admitted positions ascending (and optionally in admission order,
 //     with the best-minus-second margin of every admission).
 // The block has one thread per pool slot (256 for C <= 256, else 512). A launch for
@@ -119,6 +119,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
                                                     const __grid_constant__ Prof prof) {
   __shared__ SelSmall<NT> sh;
   extern __shared__ __align__(16) uint8_t dyn[];
+  wait_previous_kernel();   // mu and sigma come from the score kernel launched before
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
 
@@ -144,15 +145,18 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   uint32_t* keys = P.keys + keys_off + u.mu_off;
   const int h = P.pool_kernel / 2;
 
-  // shared memory: [ big | spos | cpos | inv | hist0 ]; `big` holds in turn the pooling
-  // tiles, the radix histogram and the staged candidate keys
+  // shared memory: [ big | cpos | ckey | spos | skey | inv | hist0 ]; `big` holds in
+  // turn the pooling tiles, the radix histogram and tie list, the threshold bin's
+  // (key, position) pairs, and the staged candidate keys
   uint8_t* big = dyn;
   uint4* krow = reinterpret_cast<uint4*>(big);                                  // [NT][kChunks]
   uint32_t* hist12 = reinterpret_cast<uint32_t*>(big);                          // [kBins] later passes
   float* tmu = reinterpret_cast<float*>(big);                                   // pooling tiles
-  int32_t* spos = reinterpret_cast<int32_t*>(big + kChunks * NT * sizeof(uint4));
-  int32_t* cpos = spos + NT;
-  float* inv = reinterpret_cast<float*>(cpos + NT);
+  int32_t* cpos = reinterpret_cast<int32_t*>(big + kChunks * NT * sizeof(uint4));   // pool positions
+  uint32_t* ckey = reinterpret_cast<uint32_t*>(cpos + NT);                      // and their keys
+  int32_t* spos = reinterpret_cast<int32_t*>(ckey + NT);                        // sorted pool (or the
+  uint32_t* skey = reinterpret_cast<uint32_t*>(spos + NT);                      // admitted positions)
+  float* inv = reinterpret_cast<float*>(skey + NT);
   uint32_t* hist0 = reinterpret_cast<uint32_t*>(inv + NT);                      // [kBins] first pass
 
   for (int b = tid; b < kBins; b += NT) hist0[b] = 0;
@@ -413,7 +417,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
         if (i < Lc) {
           const uint32_t d = kb[j] >> 20;
           if (d > bin) {
-            cpos[atomicAdd(&sh.cnt, 1u)] = i;
+            const uint32_t e = atomicAdd(&sh.cnt, 1u);
+            cpos[e] = i;
+            ckey[e] = kb[j];
           } else if (d == bin) {
             const uint32_t e = atomicAdd(&sh.ncand, 1u);
             if (e < kCandCap<NT>()) {
@@ -445,7 +451,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     for (uint32_t e = tid; e < ncand; e += NT) {
       const uint32_t k = cand_k[e];
       if (k > T) {
-        cpos[atomicAdd(&sh.cnt, 1u)] = cand_p[e];
+        const uint32_t n = atomicAdd(&sh.cnt, 1u);
+        cpos[n] = cand_p[e];
+        ckey[n] = k;
       } else if (k == T) {
         const uint32_t q = atomicAdd(&sh.teq, 1u);
         if (q < kTieCap) ties[q] = cand_p[e];
@@ -464,7 +472,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
         const int i = i0 + j * NT + tid;
         if (i < Lc) {
           if (kb[j] > T) {
-            cpos[atomicAdd(&sh.cnt, 1u)] = i;
+            const uint32_t n = atomicAdd(&sh.cnt, 1u);
+            cpos[n] = i;
+            ckey[n] = kb[j];
           } else if (kb[j] == T) {
             const uint32_t e = atomicAdd(&sh.teq, 1u);
             if (e < kTieCap) ties[e] = i;
@@ -496,7 +506,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       const int pos = ties[e];
       uint32_t rank = 0;
       for (uint32_t f = 0; f < n_eq; ++f) rank += (ties[f] < pos);
-      if (rank < needT) cpos[n_above + rank] = pos;
+      if (rank < needT) {
+        cpos[n_above + rank] = pos;
+        ckey[n_above + rank] = T;
+      }
     }
   } else {
     // many equal keys: ordered block scan over the positions
@@ -506,24 +519,37 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       const bool f = (i < Lc) && (__ldcg(&keys[i]) == T);
       uint32_t tot;
       const uint32_t pre = block_excl_count<NT>(f, sh, &tot);
-      if (f && taken + pre < needT) cpos[n_above + taken + pre] = i;
+      if (f && taken + pre < needT) {
+        cpos[n_above + taken + pre] = i;
+        ckey[n_above + taken + pre] = T;
+      }
       taken += tot;
     }
   }
   __syncthreads();
 
-  // 4. sort the pool by position, normalise, stage keys and inverse norms
+  // 4. the pool with its keys. Below 2^23 positions the greedy breaks ties by position
+  //    itself (position and slot packed in 32 bits), so the pool stays in the order it
+  //    was collected in; beyond that the pool is sorted by position, so that "lower
+  //    slot" means "lower position". Normalise, stage keys and inverse norms.
+  const bool packed = Lc < (1 << 23);   // position << 9 | slot stays below 0xFFFFFFFF
+  const int32_t* ppos = packed ? cpos : spos;
+  const uint32_t* pkey = packed ? ckey : skey;
   if (tid < C) {
     const int pos = cpos[tid];
-    int rank = 0;
-    for (int c = 0; c < C; ++c) rank += (cpos[c] < pos);
-    spos[rank] = pos;
-    atomicMax(&sh.maxkey, __ldcg(&keys[pos]));
+    const uint32_t key = ckey[tid];
+    if (!packed) {
+      int rank = 0;
+      for (int c = 0; c < C; ++c) rank += (cpos[c] < pos);
+      spos[rank] = pos;
+      skey[rank] = key;
+    }
+    atomicMax(&sh.maxkey, key);
   }
   __syncthreads();
   const float smax = fmaxf(unord_key(sh.maxkey), P.norm_eps);
-  // candidate keys row-major in shared memory (slot order = position order); a
-  // half-warp copies one 256-byte row, coalesced
+  // candidate keys row-major in shared memory; a half-warp copies one 256-byte row,
+  // coalesced
   {
     constexpr int kRows = NT / (NT / 32 * 2);      // rows per half-warp: 8 (NT=256) or 16 (NT=512)
     uint4 xr[kRows];
@@ -532,9 +558,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       const int r = (q * (NT / 32) + warp) * 2 + (lane >> 4);
       xr[q] = make_uint4(0, 0, 0, 0);
       if (r < C) {
-        const int pos = spos[r];
+        const int pos = ppos[r];
         if (pos >= 0 && pos < Lc) {
-          const uint4* src = reinterpret_cast<const uint4*>(P.k + (u.k_row0 + pos) * kHeadDim);
+          const uint4* src = reinterpret_cast<const uint4*>(P.k + u.k_off + pos * P.g.k_st);
           xr[q] = __ldg(src + (lane & 15));
         } else if (P.err) {
           atomicOr(P.err, kErrCheck);   // never read outside the unit's keys
@@ -565,13 +591,18 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   //    warp*32 + 16*(t>>1) + g + 8*(t&1); the warp's 32 candidate keys stay in
   //    registers as mma.m16n8k16 A fragments, and every admission computes the
   //    32 dot products with the admitted key by 16 tensor-core MMAs (bf16 products,
-  //    fp32 accumulation) with that key replicated in the 8 columns of B.
+  //    fp32 accumulation) with that key replicated in the 8 columns of B. The
+  //    argmax takes the largest value, then the smallest tie key (position << 9 |
+  //    slot, or the slot of a sorted pool): ties go to the lower position.
   const int g = lane >> 2, tq = lane & 3;
   const int slot = warp * 32 + 16 * (tq >> 1) + g + 8 * (tq & 1);
   bool active = slot < C;
   float corr = 0.f;
-  const float my_st = active ? __fdiv_rn(unord_key(__ldcg(&keys[spos[slot]])), smax) : 0.f;
+  const float my_st = active ? __fdiv_rn(unord_key(pkey[slot]), smax) : 0.f;
   const float my_inv = active ? inv[slot] : 0.f;
+  const uint32_t my_tie = !active ? 0xFFFFFFFFu
+                                  : (packed ? (static_cast<uint32_t>(ppos[slot]) << 9) | static_cast<uint32_t>(slot)
+                                            : static_cast<uint32_t>(slot));
   const uint32_t* kw = reinterpret_cast<const uint32_t*>(krow);   // 64 words per row
   uint32_t afr[2][8][4];
 #pragma unroll
@@ -587,34 +618,37 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   }
   int32_t* order = P.order ? P.order + out_off + u.unit * B : nullptr;
   float* margins = P.margins ? P.margins + out_off + u.unit * B : nullptr;
+  // admitted positions in admission order (the pool's other pair of arrays is free)
+  int32_t* adm = packed ? spos : cpos;
   for (int t = 0; t < nsel; ++t) {
     const uint32_t key = active ? ord_key(fmaf(lambda2, corr, my_st)) : 0u;
     const uint32_t wmax = __reduce_max_sync(0xffffffffu, key);
-    const uint32_t wslot = __reduce_min_sync(0xffffffffu, (active && key == wmax) ? slot : 0xFFFFFFFFu);
+    const uint32_t wtie = __reduce_min_sync(0xffffffffu, (active && key == wmax) ? my_tie : 0xFFFFFFFFu);
     // the runner-up only feeds the margins output
-    const uint32_t wsec =
-        margins ? __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(slot) == wslot ? 0u : key) : 0u;
+    const uint32_t wsec = margins ? __reduce_max_sync(0xffffffffu, my_tie == wtie ? 0u : key) : 0u;
     if (lane == 0) {
       sh.red[t & 1][warp][0] = wmax;
-      sh.red[t & 1][warp][1] = wslot;
+      sh.red[t & 1][warp][1] = wtie;
       sh.red[t & 1][warp][2] = wsec;
     }
     __syncthreads();
     // every warp reduces the NT/32 warp results itself (lane w holds warp w's)
     const bool hold = lane < NT / 32;
     const uint32_t k_l = hold ? sh.red[t & 1][lane][0] : 0u;
-    const uint32_t sl_l = hold ? sh.red[t & 1][lane][1] : 0xFFFFFFFFu;
+    const uint32_t tie_l = hold ? sh.red[t & 1][lane][1] : 0xFFFFFFFFu;
     const uint32_t best = __reduce_max_sync(0xffffffffu, k_l);
-    const uint32_t bslot = __reduce_min_sync(0xffffffffu, k_l == best ? sl_l : 0xFFFFFFFFu);
+    const uint32_t btie = __reduce_min_sync(0xffffffffu, k_l == best ? tie_l : 0xFFFFFFFFu);
     uint32_t sec = 0;
     if (margins) {
       const uint32_t k2_l = hold ? sh.red[t & 1][lane][2] : 0u;
       // runner-up: the other warps' best and the winning warp's second
-      sec = __reduce_max_sync(0xffffffffu, (k_l == best && sl_l == bslot) ? k2_l : max(k_l, k2_l));
+      sec = __reduce_max_sync(0xffffffffu, (k_l == best && tie_l == btie) ? k2_l : max(k_l, k2_l));
     }
-    const int js = static_cast<int>(bslot);
+    const int js = static_cast<int>(packed ? (btie & 511u) : btie);
     if (tid == 0) {
-      if (order) order[t] = spos[js];
+      const int pos = packed ? static_cast<int>(btie >> 9) : ppos[js];
+      adm[t] = pos;
+      if (order) order[t] = pos;
       if (margins) margins[t] = sec ? unord_key(best) - unord_key(sec) : INFINITY;
     }
     if (slot == js) active = false;
@@ -660,16 +694,15 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     if (active) corr = fmaxf(corr, dot * my_inv * inv[js]);
   }
 
-  // 6. admitted positions in ascending order, then -1
-  // slot s is admitted iff its owner went inactive; mark, then rank in slot order
+  // 6. admitted positions in ascending order (rank among the nsel admissions), then -1
   __syncthreads();
-  if (slot < C) cpos[slot] = active ? 0 : 1;
-  __syncthreads();
-  const bool sel = tid < C && cpos[tid] != 0;
-  uint32_t tot;
-  const uint32_t rank = block_excl_count<NT>(sel, sh, &tot);
   int32_t* out = P.indices + out_off + u.unit * B;
-  if (sel) out[rank] = spos[tid];
+  for (int e = tid; e < nsel; e += NT) {
+    const int pos = adm[e];
+    int rank = 0;
+    for (int f = 0; f < nsel; ++f) rank += (adm[f] < pos);
+    out[rank] = pos;
+  }
   for (int r = nsel + tid; r < B; r += NT) out[r] = -1;
   if (order)
     for (int r = nsel + tid; r < B; r += NT) order[r] = -1;
@@ -679,8 +712,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
 
 template <int NT>
 constexpr size_t select_smem() {
-  // candidate keys (also reused for the pooling tiles and the histogram) + 3 arrays
-  return kChunks * NT * sizeof(uint4) + 3 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
+  // candidate keys (also reused for the pooling tiles, the histograms, the threshold
+  // bin's keys and the tie list) + 5 arrays + the first-digit histogram
+  return kChunks * NT * sizeof(uint4) + 5 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
 }
 static_assert(kChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histogram fits");
 static_assert(kChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
@@ -705,15 +739,14 @@ cudaError_t launch_select_grid(const kve_plan& plan, const SelectParams& p, cons
     cudaError_t e = cudaFuncSetAttribute(select_kernel<256, Prof>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    select_kernel<256, Prof><<<grid, 256, smem, stream>>>(p, prof);
+    return launch_after_previous(select_kernel<256, Prof>, grid, dim3(256), smem, stream, p, prof);
   } else {
     constexpr size_t smem = select_smem<512>();
     cudaError_t e = cudaFuncSetAttribute(select_kernel<512, Prof>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
     if (e != cudaSuccess) return e;
-    select_kernel<512, Prof><<<grid, 512, smem, stream>>>(p, prof);
+    return launch_after_previous(select_kernel<512, Prof>, grid, dim3(512), smem, stream, p, prof);
   }
-  return cudaGetLastError();
 }
 
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream) {

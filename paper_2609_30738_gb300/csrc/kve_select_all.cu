@@ -71,6 +71,7 @@ __device__ __forceinline__ void block_best(uint32_t key, uint32_t idx, AllSmall&
 }
 
 __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid_constant__ SelectParams P) {
+  wait_previous_kernel();   // mu and sigma come from the score kernel launched before
   __shared__ AllSmall sh;
   extern __shared__ __align__(16) uint8_t dyn[];
   const int tid = threadIdx.x;
@@ -89,7 +90,8 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
   const float* sg = P.sigma + u.mu_off;
   float* st = reinterpret_cast<float*>(P.keys + u.mu_off);   // s~ per candidate
   float2* cinv = reinterpret_cast<float2*>(P.corr) + u.mu_off;   // (corr_i, 1 / |k_i|)
-  const uint16_t* kb = P.k + u.k_row0 * kHeadDim;
+  const uint16_t* kb = P.k + u.k_off;   // key i at kb + i * k_st
+  const int64_t kst = P.g.k_st;
   const int h = P.pool_kernel / 2;
 
   float* v = reinterpret_cast<float*>(dyn);                         // [kMaxAllCand]
@@ -123,7 +125,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
     st[i] = s;
     v[i] = s;                     // corr = 0: s~ + lambda2 * 0
     applied[i] = 0;
-    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kHeadDim);
+    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kst);
     float ss = 0.f;
     for (int c = 0; c < kHeadDim / 8; ++c) {
       const uint4 x = __ldg(ki + c);
@@ -159,14 +161,14 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
   // kRefreshGroup admissions per pass over the candidate's row (each dot keeps the
   // element order of a plain loop); staged admitted keys come from shared memory
   auto refresh = [&](int i, int t) {
-    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kHeadDim);
+    const uint4* ki = reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(i) * kst);
     const float2 ci = cinv[i];
     const float inv_i = ci.y;
     float cmax = ci.x;
     // admitted key a, chunk c: staged in shared memory or read from K
     auto adm_chunk = [&](int a, int c) -> uint4 {
       return a < kAdmStage ? admk[a * kAdmStride + c]
-                           : __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(adm[a]) * kHeadDim) + c);
+                           : __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(adm[a]) * kst) + c);
     };
     int a0 = applied[i];
     for (; a0 + kRefreshGroup <= t; a0 += kRefreshGroup) {
@@ -213,7 +215,8 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
   // admitted keys a_lo .. t-1 form the B operand, 16 per pass (two n-tiles), where
   // a_lo is the smallest count applied among the warp's stale bests; a dot against
   // an admission already applied leaves the running maximum unchanged.
-  const uint32_t* kw32 = reinterpret_cast<const uint32_t*>(kb);          // 64 words per row
+  const uint32_t* kw32 = reinterpret_cast<const uint32_t*>(kb);          // row i at kw32 + i * kst / 2
+  const int64_t kst32 = kst / 2;
   const uint32_t* admw = reinterpret_cast<const uint32_t*>(admk);        // 4 * kAdmStride words per row
   auto refresh_stale_bests = [&](int t) {
     const bool stale = my_idx != 0xFFFFFFFFu && applied[my_idx] < t;
@@ -232,7 +235,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
 #pragma unroll
         for (int hh = 0; hh < 2; ++hh) {
           const int src = 16 * m + 8 * hh + g;
-          ra[m][hh] = kw32 + static_cast<int64_t>(__shfl_sync(0xffffffffu, row, src)) * (kHeadDim / 2);
+          ra[m][hh] = kw32 + static_cast<int64_t>(__shfl_sync(0xffffffffu, row, src)) * kst32;
           ir[m][hh] = __shfl_sync(0xffffffffu, ci.y, src);
         }
       for (int a0 = a_lo; a0 < t; a0 += 16) {
@@ -252,7 +255,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
           bv[n] = an < t;
           rb[n] = !bv[n] ? kw32
                          : (an < kAdmStage ? admw + an * (4 * kAdmStride)
-                                           : kw32 + static_cast<int64_t>(adm[an]) * (kHeadDim / 2));
+                                           : kw32 + static_cast<int64_t>(adm[an]) * kst32);
         }
 #pragma unroll
         for (int s8 = 0; s8 < kHeadDim / 16; ++s8) {
@@ -343,7 +346,7 @@ __global__ void __launch_bounds__(kAllThreads, 1) select_all_kernel(const __grid
     }
     if (t < kAdmStage && tid < kHeadDim / 8)
       admk[t * kAdmStride + tid] =
-          __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(bi) * kHeadDim) + tid);
+          __ldg(reinterpret_cast<const uint4*>(kb + static_cast<int64_t>(bi) * kst) + tid);
     __syncthreads();
     if (tid == (bi % kAllThreads)) rescan();
     if (margins) {
@@ -401,8 +404,8 @@ cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaS
   cudaError_t e = cudaFuncSetAttribute(select_all_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  select_all_kernel<<<static_cast<unsigned>(plan.geo.n_units), kAllThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  return launch_after_previous(select_all_kernel, dim3(static_cast<unsigned>(plan.geo.n_units)),
+                               dim3(kAllThreads), smem, stream, p);
 }
 
 }  // namespace kve

@@ -19,7 +19,7 @@ KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 
 # Names declared in include/kv_evict.h.
 EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_destroy",
-           "kv_evict_plan_set_debug",
+           "kv_evict_plan_set_debug", "kv_evict_plan_set_kv_strides",
            "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
            "kv_evict_select_profiles_workspace", "kv_evict_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
@@ -60,6 +60,7 @@ def _lib():
         lib.kv_evict_plan_destroy.argtypes = [vp]
         lib.kv_evict_plan_destroy.restype = None
         lib.kv_evict_plan_set_debug.argtypes = [vp, ctypes.c_uint64, i32]
+        lib.kv_evict_plan_set_kv_strides.argtypes = [vp, vp, vp]
         lib.kv_evict_score.argtypes = [vp] * 7
         lib.kv_evict_select.argtypes = [vp] * 11
         lib.kv_evict_select_noalloc.argtypes = [vp] * 10
@@ -71,6 +72,7 @@ def _lib():
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
         lib.kv_evict_strerror.restype = ctypes.c_char_p
         for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_set_debug",
+                     "kv_evict_plan_set_kv_strides",
                      "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc",
                      "kv_evict_select_profiles", "kv_evict_select_profiles_workspace", "kv_evict_gather",
                      "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
@@ -120,7 +122,8 @@ class Plan:
     kv_evict_plan_ex with KVE_PLAN_PER_QUERY_HEAD when per_query_head) for a
     configuration and the prefix lengths of the requests."""
 
-    def __init__(self, spec: dict, seq_lens, layer_budgets=None, per_query_head: bool = False):
+    def __init__(self, spec: dict, seq_lens, layer_budgets=None, per_query_head: bool = False,
+                 k_strides=None, v_strides=None):
         lib = _lib()
         self.spec = dict(spec)
         self.seq_lens = [int(x) for x in seq_lens]
@@ -148,6 +151,8 @@ class Plan:
                    "kv_evict_plan_layered")
         self._h = handle
         self.workspace_bytes = ws.value
+        if k_strides is not None or v_strides is not None:
+            self.set_kv_strides(k_strides, v_strides)
 
     def __del__(self):
         h = getattr(self, "_h", None)
@@ -168,6 +173,16 @@ class Plan:
     @property
     def score_elems(self) -> int:
         return self.spec["num_layers"] * self.unit_heads * sum(self.seq_lens)
+
+    def set_kv_strides(self, k_strides=None, v_strides=None):
+        """kv_evict_plan_set_kv_strides: element strides (layer, KV head, token) of k
+        and v, None for the dense default. For a torch tensor viewed as
+        [N_L][Hkv][SL][d], pass t.stride()[:3]."""
+        ks = None if k_strides is None else np.ascontiguousarray(k_strides, dtype=np.int64)
+        vs = None if v_strides is None else np.ascontiguousarray(v_strides, dtype=np.int64)
+        _check(_lib().kv_evict_plan_set_kv_strides(self._h, None if ks is None else ks.ctypes.data,
+                                                    None if vs is None else vs.ctypes.data),
+               "kv_evict_plan_set_kv_strides")
 
     def set_debug(self, wait_limit_ns: int, fault: int = 0):
         _check(_lib().kv_evict_plan_set_debug(self._h, int(wait_limit_ns), int(fault)),

@@ -244,3 +244,27 @@ def test_noalloc_size_limit_counts_units_per_layer_without_gpu():
     big = K.Plan(spec, [16385])
     assert lib.kv_evict_select_noalloc(big._h, fake, fake, fake, lam.ctypes.data, lam.ctypes.data,
                                        fake, None, None, None) == K.KVE_EINVAL
+
+
+def test_kv_strides_validation_without_gpu():
+    """kv_evict_plan_set_kv_strides: strides in elements (layer, KV head, token), each a
+    multiple of 8 and below 2^37, the token stride at least d; NULL restores the dense
+    layout; a refused call leaves the plan as it was."""
+    _need_lib()
+    from paper_2609_30738_gb300 import kv_evict as K
+    SL, Hkv, d = 2048 + 777, 8, 128
+    p = K.Plan(_spec(), [2048, 777])
+    p.set_kv_strides((SL * Hkv * d, d, Hkv * d), (Hkv * SL * 2 * d, SL * 2 * d, 2 * d))
+    p.set_kv_strides(None, None)
+    p.set_kv_strides((Hkv * SL * d, SL * d, d))
+    for bad in [(SL * Hkv * d, d, 64),            # token stride below d
+                (SL * Hkv * d + 4, d, Hkv * d),    # not a multiple of 8 elements
+                (-8, d, Hkv * d),
+                (1 << 37, d, Hkv * d)]:
+        with pytest.raises(K.KvEvictError) as e:
+            p.set_kv_strides(bad, None)
+        assert e.value.status == K.KVE_EINVAL
+        with pytest.raises(K.KvEvictError) as e:
+            p.set_kv_strides(None, bad)
+        assert e.value.status == K.KVE_EINVAL
+    assert K.library().kv_evict_plan_set_kv_strides(None, None, None) == K.KVE_EINVAL

@@ -362,6 +362,36 @@ def test_every_candidate_greedy(L, B, lams):
     _check_units(spec, batch, plan, bufs, lam, _all_units(spec, batch["seq_lens"]))
 
 
+@pytest.mark.parametrize("cf", [4, 0])
+def test_strided_kv_layouts_equal_dense(cf):
+    """k and v read in place from a serving engine's layouts (plan strides): a
+    token-major key cache [N_L][SL][Hkv][d] and a value cache whose rows are padded
+    to 2d elements. Every output -- mu, sigma, the selection with its order and
+    margins, the compact cache -- equals the dense-layout call bit for bit, with the
+    pooled selector (factor 4) and the every-candidate selector (factor 0)."""
+    from paper_2609_30738_gb300 import kv_evict as K
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=24, candidate_factor=cf,
+                  seq_lens=[700, 1500, 300])
+    batch = synth.make_batch(spec, seed=61)
+    plan, bufs, (q, k, v), lam = _run(spec, batch)
+    N_L, Hkv, d, SL = spec["num_layers"], spec["num_kv_heads"], spec["head_dim"], sum(batch["seq_lens"])
+    kt = k.permute(0, 2, 1, 3).contiguous()                     # [N_L][SL][Hkv][d]
+    vbuf = torch.full((N_L, Hkv, SL, 2 * d), 7.0, dtype=torch.bfloat16, device=DEV)
+    vbuf[..., :d] = v
+    k_str = (kt.stride(0), kt.stride(2), kt.stride(1))          # (layer, head, token)
+    v_str = (vbuf.stride(0), vbuf.stride(1), vbuf.stride(2))
+    assert k_str == (SL * Hkv * d, d, Hkv * d) and v_str[2] == 2 * d
+    plan2 = K.Plan(spec, batch["seq_lens"], k_strides=k_str, v_strides=v_str)
+    bufs2 = K.Buffers(plan2)
+    plan2.score(q, kt, bufs2.mu, bufs2.sigma, bufs2.ws)
+    plan2.select(bufs2.mu, bufs2.sigma, kt, lam[0], lam[1], bufs2.indices, bufs2.ws, bufs2.order,
+                 bufs2.margins)
+    plan2.gather(kt, vbuf, bufs2.indices, bufs2.k_out, bufs2.v_out)
+    assert plan2.status(bufs2.ws) == K.KVE_OK
+    for name in ("mu", "sigma", "indices", "order", "margins", "k_out", "v_out"):
+        assert torch.equal(getattr(bufs, name), getattr(bufs2, name)), name
+
+
 def test_repeatable_bitwise():
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], seq_lens=[3000, 700])
     batch = synth.make_batch(spec, seed=11)
