@@ -46,8 +46,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "6593b248e96b4d98f638c81c75750ae26af939cef30a1c7eb39fbcb49690d658",
-                 "bytes_per_launch": 2178506496 + 75100672}
+SCORE_TRAFFIC = {"source_sha256": "11bb2d9436bf0db49e8069c6c29b7524323b6dfe53d05699dec9b583a21b3653",
+                 "bytes_per_launch": 2172357376 + 74841600}
 
 
 def _score_source_sha():
