@@ -395,6 +395,29 @@ def run_ours(args):
         raise RuntimeError("device-side wait timed out in the timed region")
     elapsed = _max_over_ranks(elapsed, world, dev)
 
+    # the score pass with the window rows' attention output (kv_evict_score_attn): the
+    # same K stream plus V, timed alone beside the plain score kernel
+    window = None
+    if batch is not None and args.attn_steps > 0:
+        attn_ws = torch.empty(plan.score_attn_workspace(), dtype=torch.uint8, device=dev)
+        o_win = torch.empty_like(q)
+        with torch.cuda.stream(stream):
+            plan.score_attn(q, k, v, bufs.mu, bufs.sigma, o_win, bufs.ws, attn_ws, stream)
+        if plan.status(bufs.ws, stream) != K.KVE_OK:
+            raise RuntimeError("device-side wait timed out in the window-output pass")
+        wa, wb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        wa.record(stream)
+        for _ in range(args.attn_steps):
+            plan.score_attn(q, k, v, bufs.mu, bufs.sigma, o_win, bufs.ws, attn_ws, stream)
+        wb.record(stream)
+        torch.cuda.synchronize()
+        attn_s = wa.elapsed_time(wb) / 1e3 / args.attn_steps
+        kv_bytes = 2 * sum(N_L * Hkv * Lr * d * 2 for Lr in seq)
+        window = {"score_attn_ms": attn_s * 1e3, "score_ms": score_s * 1e3,
+                  "kv_read_bytes": kv_bytes, "kv_read_gbs": kv_bytes / attn_s / 1e9,
+                  "attn_ws_bytes": int(attn_ws.numel())}
+        del attn_ws, o_win
+
     # end to end through the public API with host buffers (pinned), copies inside.
     # A one-request call is evicted in chunks of layers, one plan per chunk: the copy
     # stream brings in chunk c + 1 while the compute stream scores, selects and
@@ -453,7 +476,7 @@ def run_ours(args):
                          "algorithmic_bytes_per_launch": k_read,
                          "secondary_bytes_per_launch": secondary},
             "gpu_launches": 3 * args.steps,
-            "clocks": clocks, "cpu_baseline": cpu, "e2e": e2e}
+            "clocks": clocks, "cpu_baseline": cpu, "e2e": e2e, "window_output": window}
     print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -572,6 +595,8 @@ def main():
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="layer chunks of the end-to-end step (copy of chunk c+1 beside compute of c)")
     ap.add_argument("--cpu-units", type=int, default=128)
+    ap.add_argument("--attn-steps", type=int, default=10,
+                    help="launches of the score pass with the window output, timed beside the step")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling only: fewer layers than the workload (0 = all)")
     args = ap.parse_args()

@@ -158,6 +158,27 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win,
                           const uint16_t* k, float* mu, float* sigma, void* ws,
                           void* stream);
 
+/* Steps 1-2 as kv_evict_score, together with the window rows' own attention output.
+ * Section 3.2 scores the tokens with the prefill's existing attention; the window rows'
+ * attention (the last W positions of every query head) is computed here anyway, so in
+ * the same pass over the prefix the library also streams V and returns
+ *   O[r] = sum_i A[r][i] * v_i      (A of Eq. 1: causal softmax over the prefix)
+ * for every window row, and a caller's prefill can skip attention for those rows.
+ * o_win has q_win's layout, [N_L][n_req][Hq][W][d] bf16 (with KVE_PLAN_PER_QUERY_HEAD
+ * the same). v follows the plan's v strides. mu and sigma are those of kv_evict_score.
+ * Precision: A enters the value product as bf16 (relative error <= 2^-8 per
+ * probability), accumulated in fp32, and O is rounded to bf16 once, so
+ * |O - O_exact| <= 2^-8 (sum_i A[r][i] |v_i| + |O|) elementwise. attn_ws is a
+ * second scratch buffer (256-byte aligned) of kv_evict_score_attn_workspace bytes
+ * (fp32 partial outputs, 64 KB per score work item). v must be 128-byte aligned. */
+kve_status kv_evict_score_attn(const kve_plan* plan, const uint16_t* q_win,
+                               const uint16_t* k, const uint16_t* v, float* mu,
+                               float* sigma, uint16_t* o_win, void* ws,
+                               void* attn_ws, void* stream);
+
+/* *bytes = the attn_ws size of kv_evict_score_attn for this plan. */
+kve_status kv_evict_score_attn_workspace(const kve_plan* plan, size_t* bytes);
+
 /* Step 3: pooling (Section 3.1), base score (Eq. 2), top factor*B candidate pool
  * (Section 3.2), normalisation (Eq. 5, denominator clamped to norm_eps), greedy
  * admission by s~ + lambda2 * corr(i, S) (Eq. 4, Eq. 5) with ties broken towards

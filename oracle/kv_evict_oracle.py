@@ -21,6 +21,8 @@ float64 from the bf16-decoded inputs, in the paper's order:
   greedy_mmr         Eq. 5: S <- S + argmax_{i not in S}(s~_i + lambda2 corr(i, S)),
                      first admission argmax s~, until |S| = B.
   gather             Section 1: the layer keeps B entries (plus the window).
+  window_output      Section 3.2 ("uses existing attention"): the window rows' own
+                     attention output O[r] = sum_i A[r, i] v_i, from the same A as Eq. 1.
   depth_profile      Eq. 6: a(l) = c0 + c1 t + c2 t^2, t = l/(N_L - 1),
                      lambda = sinh(a); Global / Segments / Curve.
 
@@ -248,6 +250,14 @@ def select_unit(mu: np.ndarray, sigma: np.ndarray, keys: np.ndarray, L: int, W: 
     steps = greedy_mmr(s_tilde, keys, pool, lambda2, B, follow=follow)
     idx = np.sort(np.array([st["pick"] for st in steps], dtype=np.int64))
     return dict(indices=idx, steps=steps, pool=pool, s_tilde=s_tilde, cut_margin=cut_margin)
+
+
+def window_output(A: np.ndarray, v: np.ndarray) -> np.ndarray:
+    """The attention output of the window rows: O[r] = sum_i A[r, i] v_i over the
+    prefix (A from window_attention: causal softmax rows, 0 where masked). Section 3.2
+    scores tokens with the prefill's existing attention; these rows are that
+    attention's output for the last W positions of every query head."""
+    return A @ v
 
 
 def score_unit(q: np.ndarray, k: np.ndarray, L: int, W: int, G: int):

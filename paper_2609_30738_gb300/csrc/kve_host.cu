@@ -54,15 +54,17 @@ bool encode_rows(CUtensorMap* map, const void* base, int64_t rows) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// k viewed as a 4-D tensor (d, token, KV head, layer) with the plan's element strides;
-// boxes of 64 elements x 128 tokens with the 128-byte swizzle, tokens past SL read as zero.
-bool encode_keys(CUtensorMap* map, const void* base, const kve::Geometry& g) {
+// k (or v) viewed as a 4-D tensor (d, token, KV head, layer) with the plan's element
+// strides; boxes of 64 elements x 128 tokens with the 128-byte swizzle, tokens past SL
+// read as zero.
+bool encode_keys(CUtensorMap* map, const void* base, const kve::Geometry& g, bool values = false) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[4] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(g.total_tokens),
                         static_cast<cuuint64_t>(g.hkv), static_cast<cuuint64_t>(g.num_layers)};
-  cuuint64_t strides[3] = {static_cast<cuuint64_t>(g.k_st) * 2, static_cast<cuuint64_t>(g.k_sh) * 2,
-                           static_cast<cuuint64_t>(g.k_sl) * 2};
+  const int64_t st = values ? g.v_st : g.k_st, sh = values ? g.v_sh : g.k_sh, sl = values ? g.v_sl : g.k_sl;
+  cuuint64_t strides[3] = {static_cast<cuuint64_t>(st) * 2, static_cast<cuuint64_t>(sh) * 2,
+                           static_cast<cuuint64_t>(sl) * 2};
   cuuint32_t box[4] = {64, 128, 1, 1};
   cuuint32_t estr[4] = {1, 1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
@@ -261,17 +263,25 @@ kve_status kv_evict_plan_set_debug(kve_plan* plan, uint64_t wait_limit_ns, int32
   return KVE_OK;
 }
 
-kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, float* mu,
-                          float* sigma, void* ws, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The score step, with the window output when v is given (o_win, attn_ws then too).
+kve_status score_impl(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, const uint16_t* v,
+                      float* mu, float* sigma, uint16_t* o_win, void* ws, void* attn_ws, void* stream) {
   if (!plan || !q_win || !k || !mu || !sigma || !ws) return KVE_EINVAL;
   if (!aligned(q_win, 128) || !aligned(k, 128) || !aligned(mu, 16) || !aligned(sigma, 16) || !aligned(ws, 256))
+    return KVE_EINVAL;
+  if (v && (!o_win || !attn_ws || !aligned(v, 128) || !aligned(o_win, 16) || !aligned(attn_ws, 256)))
     return KVE_EINVAL;
   const kve::Geometry& g = plan->geo;
   const int sms = device_sms();
   if (sms <= 0) return KVE_ECUDA;
-  CUtensorMap tm_q, tm_k;
+  CUtensorMap tm_q, tm_k, tm_v;
   const int64_t q_rows = static_cast<int64_t>(g.num_layers) * g.n_req * g.hq * g.window;
   if (!encode_rows(&tm_q, q_win, q_rows) || !encode_keys(&tm_k, k, g)) return KVE_ECUDA;
+  if (v && !encode_keys(&tm_v, v, g, true)) return KVE_ECUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint8_t* w = static_cast<uint8_t*>(ws);
   if (cudaMemsetAsync(w, 0, plan->ws.clear_end, st) != cudaSuccess) return KVE_ECUDA;
@@ -287,10 +297,35 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uin
   p.counts = reinterpret_cast<uint32_t*>(w + plan->ws.counts);
   p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
   p.beta = reinterpret_cast<unsigned long long*>(w + plan->ws.beta);
+  p.o_part = static_cast<float*>(attn_ws);
   const int64_t ctas = std::min<int64_t>(sms, g.n_items);
   p.lag = score_lag(g, ctas);
-  return kve::launch_score(*plan, tm_q, tm_k, p, static_cast<int>(ctas), st) == cudaSuccess ? KVE_OK
-                                                                                        : KVE_ECUDA;
+  if (kve::launch_score(*plan, tm_q, tm_k, v ? &tm_v : nullptr, p, static_cast<int>(ctas), st) != cudaSuccess)
+    return KVE_ECUDA;
+  if (v && kve::launch_attn_finish(*plan, p.o_part, o_win, st) != cudaSuccess) return KVE_ECUDA;
+  return KVE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, float* mu,
+                          float* sigma, void* ws, void* stream) {
+  return score_impl(plan, q_win, k, nullptr, mu, sigma, nullptr, ws, nullptr, stream);
+}
+
+kve_status kv_evict_score_attn(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k,
+                               const uint16_t* v, float* mu, float* sigma, uint16_t* o_win, void* ws,
+                               void* attn_ws, void* stream) {
+  if (!v) return KVE_EINVAL;
+  return score_impl(plan, q_win, k, v, mu, sigma, o_win, ws, attn_ws, stream);
+}
+
+kve_status kv_evict_score_attn_workspace(const kve_plan* plan, size_t* bytes) {
+  if (!plan || !bytes) return KVE_EINVAL;
+  *bytes = align_up(static_cast<size_t>(plan->geo.n_items) * kMaxRows * kHeadDim * sizeof(float), 256);
+  return KVE_OK;
 }
 
 }  // extern "C"

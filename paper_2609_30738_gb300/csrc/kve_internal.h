@@ -131,6 +131,7 @@ struct ScoreParams {
   uint32_t* counts;
   float2* partial;
   unsigned long long* beta;   // low word: beta bits, high word: 1 once written
+  float* o_part;              // window output: fp32 [n_items][kMaxRows][d] per column item
 };
 
 struct SelectParams {
@@ -220,8 +221,12 @@ cudaError_t launch_after_previous(void (*fn)(KArgs...), dim3 grid, dim3 block, s
 }
 
 // Kernel launchers (defined next to their kernels).
+// tm_v = null: the plain score kernel; otherwise the variant that also accumulates the
+// window rows' attention output into p.o_part (then launch_attn_finish).
 cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                         const ScoreParams& p, int ctas, cudaStream_t stream);
+                         const CUtensorMap* tm_v, const ScoreParams& p, int ctas, cudaStream_t stream);
+cudaError_t launch_attn_finish(const kve_plan& plan, const float* o_part, uint16_t* o_win,
+                               cudaStream_t stream);
 cudaError_t launch_select(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_select_all(const kve_plan& plan, const SelectParams& p, cudaStream_t stream);
 cudaError_t launch_select_profiles(const kve_plan& plan, const SelectParams& p, const ProfileTable& table,

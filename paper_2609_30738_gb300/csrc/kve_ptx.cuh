@@ -187,7 +187,21 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return d;
 }
 
-// Instruction descriptor of kind::f16: bf16 x bf16 -> fp32, both K-major.
+// Shared-memory matrix descriptor for an MN-major operand with the 128-byte swizzle: a
+// swizzle atom is 8 K-rows of 128 bytes (64 MN elements); LBO = bytes from one atom to
+// the next along MN, SBO = bytes from one 8-row group to the next along K.
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // start address
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;                   // descriptor version
+  d |= static_cast<uint64_t>(2) << 61;                   // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor of kind::f16: bf16 x bf16 -> fp32, both K-major (bits 15 and
+// 16 transpose A and B to MN-major).
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4)                                  // D = f32
          | (1u << 7)                                // A = bf16

@@ -55,17 +55,37 @@ constexpr int kMergeWarp = 3;
 constexpr int kEpiWarp0 = 4;
 constexpr int kEpiWarps = 8;
 constexpr int kMergeSlots = 4;
-constexpr int kMergeBatch = 40;  // partials per bulk copy (1 KB each): a 38-item unit in one
 constexpr int kQBufs = 2;
-constexpr int kKStages = 3;      // K tiles in flight (32 KB each)
-constexpr int kAccBufs = 4;      // 4 x 128 TMEM columns
 constexpr int kItemSlots = 4;
 constexpr uint32_t kTileBytes = 128 * kHeadDim * 2;   // 32 KB: 128 rows x 128 bf16
 constexpr uint32_t kHalfBytes = kTileBytes / 2;       // one 64-element (128 B) column block
 constexpr uint32_t kTmemCols = 512;
-constexpr size_t kMergeBytes = static_cast<size_t>(kMergeBatch) * kMaxRows * sizeof(float2);
-constexpr size_t kDynSmem = (kQBufs + kKStages) * kTileBytes + kMergeBytes + 1024;
 constexpr uint32_t kIdesc = idesc_bf16_f32(128, 128);
+// O^T += V^T P^T with both operands MN-major (128-byte swizzle): instruction descriptor
+// with the A and B transpose bits, and the operand strides of a [128][128] bf16 tile in
+// two 64-column halves (16 KB apart along MN, 8-row groups 1 KB apart along K)
+constexpr uint32_t kIdescMN = kIdesc | (1u << 15) | (1u << 16);
+constexpr uint32_t kMNLbo = kHalfBytes;
+constexpr uint32_t kMNSbo = 1024;
+
+// Pipeline depths of the two variants. The plain kernel: 3 K stages, 4 score
+// accumulators, partials merged 40 per bulk copy. With the window output (kAttn) the
+// column pass also streams V and accumulates O^T on the tensor cores: 2 K stages (a
+// column tile's stage then holds its probabilities P^T until the O^T MMA has read
+// them), 2 V stages, 3 score accumulators and the O^T accumulator in TMEM columns
+// 384..511, and a smaller merge buffer.
+template <bool kAttn>
+struct Cfg {
+  static constexpr int kKStages = kAttn ? 2 : 3;
+  static constexpr int kVStages = kAttn ? 2 : 0;
+  static constexpr int kAccBufs = kAttn ? 3 : 4;
+  static constexpr int kMergeBatch = kAttn ? 8 : 40;   // partials per bulk copy (1 KB each)
+  static constexpr size_t kMergeBytes = static_cast<size_t>(kMergeBatch) * kMaxRows * sizeof(float2);
+  static constexpr size_t kDynSmem = (kQBufs + kKStages + kVStages) * kTileBytes + kMergeBytes + 1024;
+};
+constexpr int kMaxKStages = 3;
+constexpr int kMaxAccBufs = 4;
+constexpr uint32_t kOCol = 384;   // TMEM column of the O^T accumulator (window output)
 
 // One pass over one item, as the producer derives it once from the item index and
 // hands it to the other roles through the item ring (p = -1 ends the work).
@@ -98,8 +118,12 @@ struct MergeJob {
 
 struct ScoreCtl {
   uint64_t q_full[kQBufs], q_empty[kQBufs];
-  uint64_t k_full[kKStages], k_empty[kKStages];
-  uint64_t acc_full[kAccBufs], acc_empty[kAccBufs];
+  uint64_t k_full[kMaxKStages], k_empty[kMaxKStages];
+  uint64_t acc_full[kMaxAccBufs], acc_empty[kMaxAccBufs];
+  // window output only: V stages, P^T written into a K stage, the O^T accumulator
+  uint64_t v_full[2], v_empty[2];
+  uint64_t p_full[2];               // epilogue -> MMA: P^T of the tile in K stage s is written
+  uint64_t o_full, o_empty;         // MMA -> epilogue group 0 -> MMA, once per column item
   uint64_t item_full[kItemSlots], item_empty[kItemSlots];
   uint64_t pub_full[kItemSlots];    // epilogue -> sync warp, once per item
   uint64_t beta_full[kItemSlots];   // sync warp -> epilogue, once per item
@@ -143,9 +167,10 @@ __device__ __forceinline__ float2 merge_mz(float2 a, float2 b) {
 
 // ---------------------------------------------------------------- epilogue, phase 0
 
-template <bool kFull>
+template <bool kFull, bool kAttn>
 __device__ __forceinline__ bool rowstats_item(const ScoreParams& P, ScoreCtl& ctl,
                                               const ItemDesc& d, uint32_t slot, uint32_t& ai) {
+  constexpr int kAccBufs = Cfg<kAttn>::kAccBufs;
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
   const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;   // 0 or 1
@@ -263,14 +288,41 @@ __device__ __forceinline__ void col_half_values(const ScoreParams& P, const Scor
   }
 }
 
+// bf16 bits of two floats packed in one word (round to nearest even): lo in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  uint32_t d;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
+  return d;
+}
+
+// Window output: the probabilities A[r][key] = A'[r] * 2^-40 of this half's 64 rows as
+// bf16 into the P^T tile (K = the tile's 128 keys, N = the 128 rows), MN-major with the
+// 128-byte swizzle: rows 64h.. form the atom at h * 16 KB, key k's 128-byte row of it sits
+// at (k / 8) * 1024 + (k % 8) * 128, and its 16-byte chunk c (rows 8c .. 8c + 7) at
+// position c ^ (k % 8).
+__device__ __forceinline__ void write_pt_half(uint8_t* pt, int key, int h0, const float (&v)[64]) {
+  uint8_t* row = pt + (h0 >> 6) * kHalfBytes + (key >> 3) * 1024 + (key & 7) * 128;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const float* x = v + 8 * c;
+    const uint4 w = make_uint4(pack_bf16x2(x[0] * kColUnscale, x[1] * kColUnscale),
+                               pack_bf16x2(x[2] * kColUnscale, x[3] * kColUnscale),
+                               pack_bf16x2(x[4] * kColUnscale, x[5] * kColUnscale),
+                               pack_bf16x2(x[6] * kColUnscale, x[7] * kColUnscale));
+    *reinterpret_cast<uint4*>(row + ((c ^ (key & 7)) << 4)) = w;
+  }
+}
+
 // Sum and sum of squares of a half (3 fp32 operations per element with the
-// exponent's argument: the FMA pipe stays below the MUFU pipe).
-template <bool kFull>
+// exponent's argument: the FMA pipe stays below the MUFU pipe). With the window
+// output (pt != null), the half's probabilities also go to the P^T tile.
+template <bool kFull, bool kAttn>
 __device__ __forceinline__ void colsums_half(const ScoreParams& P, const ScoreCtl& ctl,
                                              const float4* nb4, uint32_t taddr, int h0, int n,
-                                             int rel, float& sum, float& sumsq) {
+                                             int rel, float& sum, float& sumsq, uint8_t* pt, int key) {
   float v[64];
   col_half_values<kFull>(P, ctl, nb4, taddr, h0, n, rel, v);
+  if constexpr (kAttn) write_pt_half(pt, key, h0, v);
   float2 c0 = make_float2(0.f, 0.f), c1 = c0, c2 = c0, c3 = c0;
   float2 q0 = c0, q1 = c0, q2 = c0, q3 = c0;
 #pragma unroll
@@ -322,9 +374,17 @@ __device__ __forceinline__ void colstats_half(const ScoreParams& P, const ScoreC
   m2 = q;
 }
 
-template <bool kFull>
+// With the window output (kAttn), every tile's probabilities go to the P^T tile in the
+// tile's K stage (kbuf + stage * 32 KB; the score MMA has finished with its K), announced
+// on p_full[stage]; at the end of the item group 0 reads the item's O^T accumulator
+// (lane = d, column = row) into o_part[item][row][d] and hands it back on o_empty. oi
+// counts the column items before this one.
+template <bool kFull, bool kAttn>
 __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ctl,
-                                              const ItemDesc& d, uint32_t slot, uint32_t& ai) {
+                                              const ItemDesc& d, uint32_t slot, uint32_t& ai,
+                                              uint8_t* kbuf, uint32_t& oi) {
+  constexpr int kAccBufs = Cfg<kAttn>::kAccBufs;
+  constexpr int kKStages = Cfg<kAttn>::kKStages;
   const int quad = (threadIdx.x >> 5) & 3;
   const int lane = threadIdx.x & 31;
   const int grp = (threadIdx.x - kEpiWarp0 * 32) >> 7;
@@ -350,11 +410,25 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     const bool two = kFull || n > 64;
     float S1 = 0.f, SS = 0.f;
 #pragma unroll 1
+    uint8_t* pt = kAttn ? kbuf + (ai % kKStages) * kTileBytes : nullptr;
     for (int h = 0; h < (two ? 2 : 1); ++h) {
       float sh, qh;
-      colsums_half<kFull>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, qh);
+      colsums_half<kFull, kAttn>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, qh, pt, tl);
       S1 += sh;
       SS += qh;
+    }
+    if constexpr (kAttn) {
+      if (!two) {
+        // rows 64..127 are past n: their probabilities are 0
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          *reinterpret_cast<uint4*>(pt + kHalfBytes + (tl >> 3) * 1024 + (tl & 7) * 128 + (c << 4)) =
+              make_uint4(0, 0, 0, 0);
+      }
+      // P^T is read by the tensor cores (async proxy) once every warp has announced it
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.p_full[ai % kKStages]);
     }
     float m2 = fmaf(-S1, S1 * inv_n, SS);
     // The one-pass form loses about (sum A'^2) * 2^-19 to rounding. It is kept while
@@ -389,6 +463,27 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
       __stcs(&P.mu[d.mu_off + key], mu);
       __stcs(&P.sigma[d.mu_off + key], sigma);
     }
+  }
+  if constexpr (kAttn) {
+    if (grp == 0) {
+      // the item's O^T (lane = d, column = row) into o_part[item][row][d]
+      if (!warp_wait(&ctl.o_full, oi & 1u, P.wait_limit_ns, &ctl.abort)) return false;
+      tc_fence_after();
+      const uint32_t taddr = ctl.tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + kOCol;
+      float* dst = P.o_part + d.p * (kMaxRows * kHeadDim) + tl;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld32(taddr + 32u * c, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) __stcg(dst + (32 * c + j) * kHeadDim, v[j]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl.o_empty);
+    }
+    ++oi;
   }
   return true;
 }
@@ -463,8 +558,10 @@ __device__ __forceinline__ bool sync_rowstats(const ScoreParams& P, ScoreCtl& ct
 // Merge warp: fold all of a unit's (m, Z) partials into beta_r = m + log2 Z and
 // publish each row's beta with its ready tag. The partials of a unit are contiguous
 // (1 KB per item) and come in by bulk copies of up to kMergeBatch items.
+template <bool kAttn>
 __device__ __forceinline__ bool merge_unit(const ScoreParams& P, ScoreCtl& ctl, const MergeJob& u,
                                            float2 (*mbuf)[kMaxRows], uint32_t& phase) {
+  constexpr int kMergeBatch = Cfg<kAttn>::kMergeBatch;
   const int lane = threadIdx.x & 31;
   const int n = P.g.n_rows;
   __threadfence();
@@ -561,18 +658,23 @@ __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ct
 
 // ---------------------------------------------------------------- kernel
 
-template <bool kFull>
+// kAttn: the window output variant (tm_v maps v; for the plain kernel tm_v is unused).
+template <bool kFull, bool kAttn>
 __global__ void __launch_bounds__(kThreads, 1)
     score_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                 const __grid_constant__ ScoreParams P) {
+                 const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ ScoreParams P) {
+  constexpr int kKStages = Cfg<kAttn>::kKStages;
+  constexpr int kAccBufs = Cfg<kAttn>::kAccBufs;
   __shared__ ScoreCtl ctl;
   extern __shared__ uint8_t dyn_smem[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(dyn_smem) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* qbuf = tiles;                             // kQBufs x 32 KB
   uint8_t* kbuf = tiles + kQBufs * kTileBytes;       // kKStages x 32 KB
+  uint8_t* vbuf = kbuf + kKStages * kTileBytes;      // kVStages x 32 KB (window output)
   // partials being merged (bulk-copy destination, 1 KB aligned)
-  float2 (*mbuf)[kMaxRows] = reinterpret_cast<float2 (*)[kMaxRows]>(kbuf + kKStages * kTileBytes);
+  float2 (*mbuf)[kMaxRows] =
+      reinterpret_cast<float2 (*)[kMaxRows]>(vbuf + Cfg<kAttn>::kVStages * kTileBytes);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -592,11 +694,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl.merge_full[i], 1);
       mbar_init(&ctl.merge_empty[i], 1);
     }
+    if constexpr (kAttn) {
+      for (int i = 0; i < Cfg<kAttn>::kVStages; ++i) {
+        mbar_init(&ctl.v_full[i], 1);
+        mbar_init(&ctl.v_empty[i], 1);
+      }
+      for (int i = 0; i < kKStages; ++i) mbar_init(&ctl.p_full[i], 4);   // the tile's 4 warps
+      mbar_init(&ctl.o_full, 1);
+      mbar_init(&ctl.o_empty, 4);                                          // group 0
+    }
     mbar_init(&ctl.merge_bar, 1);
     ctl.abort = 0;
     fence_mbar_init();
     prefetch_tensormap(&tm_q);
     prefetch_tensormap(&tm_k);
+    if (kAttn) prefetch_tensormap(&tm_v);
   }
   if (threadIdx.x < kMaxRows) {
     ctl.roww[threadIdx.x] = threadIdx.x % P.g.window;
@@ -613,9 +725,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      uint32_t it = 0, qi = 0, ki = 0;
+      uint32_t it = 0, qi = 0, ki = 0, vi = 0;
       // bit i: buffer / stage i has been loaded at least once, and the parity of its last load
-      uint32_t q_used = 0, k_used = 0, q_last = 0, k_last = 0;
+      uint32_t q_used = 0, k_used = 0, q_last = 0, k_last = 0, v_used = 0, v_last = 0;
       const uint64_t pol_keep = l2_policy_evict_last();
       const uint64_t pol_drop = l2_policy_evict_first();
       bool ok = true;
@@ -699,6 +811,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           k_used |= 1u << ks;
           k_last = (k_last & ~(1u << ks)) | (((ki / kKStages) & 1u) << ks);
           ++ki;
+          if constexpr (kAttn) {
+            if (cl.phase == 1) {
+              // the tile's values for the window output (streamed once, from HBM)
+              const uint32_t vs = vi % Cfg<kAttn>::kVStages;
+              const uint32_t vpar = (vi / Cfg<kAttn>::kVStages) & 1u;
+              if (!mbar_wait(&ctl.v_empty[vs], vpar ^ 1u, P.wait_limit_ns, &ctl.abort)) {
+                ok = false;
+                break;
+              }
+              mbar_arrive_expect_tx(&ctl.v_full[vs], kTileBytes);
+              tma_load_4d_hint(vbuf + vs * kTileBytes, &tm_v, 0, y, d.kvh, d.layer, &ctl.v_full[vs],
+                               pol_drop);
+              tma_load_4d_hint(vbuf + vs * kTileBytes + kHalfBytes, &tm_v, 64, y, d.kvh, d.layer,
+                               &ctl.v_full[vs], pol_drop);
+              v_used |= 1u << vs;
+              v_last = (v_last & ~(1u << vs)) | (vpar << vs);
+              ++vi;
+            }
+          }
         }
         if (!ok) break;
       }
@@ -709,6 +840,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if ((q_used >> i) & 1u) mbar_wait(&ctl.q_full[i], (q_last >> i) & 1u, P.wait_limit_ns, &no_abort);
       for (int i = 0; i < kKStages; ++i)
         if ((k_used >> i) & 1u) mbar_wait(&ctl.k_full[i], (k_last >> i) & 1u, P.wait_limit_ns, &no_abort);
+      for (int i = 0; i < Cfg<kAttn>::kVStages; ++i)
+        if ((v_used >> i) & 1u) mbar_wait(&ctl.v_full[i], (v_last >> i) & 1u, P.wait_limit_ns, &no_abort);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -719,6 +852,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t qaddr = smem_u32(qbuf);
       const uint32_t kaddr = smem_u32(kbuf);
       bool ok = true;
+      // window output: the O^T MMA of a column tile runs one tile behind its score MMA
+      // (its P^T must be written first); pend_* describe the tile waiting for it
+      const uint32_t vaddr = smem_u32(vbuf);
+      uint32_t vi = 0, oi = 0, pcnt[2] = {0u, 0u}, last_opar = 0;
+      int pend_ks = -1, pend_vs = 0, o_issued = 0;
+      uint32_t pend_vpar = 0;
+      bool pend_first = false;
+      auto issue_pv = [&]() -> bool {
+        if (!mbar_wait(&ctl.p_full[pend_ks], pcnt[pend_ks] & 1u, P.wait_limit_ns, &ctl.abort) ||
+            !mbar_wait(&ctl.v_full[pend_vs], pend_vpar, P.wait_limit_ns, &ctl.abort) ||
+            (pend_first && !mbar_wait(&ctl.o_empty, (oi & 1u) ^ 1u, P.wait_limit_ns, &ctl.abort)))
+          return false;
+        ++pcnt[pend_ks];
+        tc_fence_after();
+        const uint32_t va = vaddr + pend_vs * kTileBytes, pa = kaddr + pend_ks * kTileBytes;
+#pragma unroll
+        for (int j = 0; j < kHeadDim / 16; ++j)   // 16 keys per MMA: 2 KB of each operand
+          tc_mma_bf16(ctl.tmem_base + kOCol, sw128_mn_desc(va + 2048u * j, kMNLbo, kMNSbo),
+                      sw128_mn_desc(pa + 2048u * j, kMNLbo, kMNSbo), kIdescMN,
+                      (pend_first && j == 0) ? 0u : 1u);
+        tc_commit(&ctl.k_empty[pend_ks]);
+        tc_commit(&ctl.v_empty[pend_vs]);
+        pend_ks = -1;
+        return true;
+      };
       for (;;) {
         const uint32_t slot = it % kItemSlots;
         if (!mbar_wait(&ctl.item_full[slot], (it / kItemSlots) & 1u,
@@ -762,15 +920,41 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t off = ((j >> 2) * kHalfBytes + (j & 3) * 32u) >> 4;
             tc_mma_bf16(d_tmem, ad + off, bd + off, kIdesc, j > 0 ? 1u : 0u);
           }
-          tc_commit(&ctl.k_empty[ks]);
+          if (!kAttn || phase == 0) tc_commit(&ctl.k_empty[ks]);
           tc_commit(&ctl.acc_full[ab]);
           issued = 1;
           last_ab = ab;
           last_par = (ai / kAccBufs) & 1u;
+          if constexpr (kAttn) {
+            if (phase == 1) {
+              if (pend_ks >= 0 && !issue_pv()) {
+                ok = false;
+                break;
+              }
+              pend_ks = static_cast<int>(ks);
+              pend_vs = static_cast<int>(vi % Cfg<kAttn>::kVStages);
+              pend_vpar = (vi / Cfg<kAttn>::kVStages) & 1u;
+              pend_first = t == 0;
+              ++vi;
+            }
+          }
           ++ki;
           ++ai;
         }
         if (!ok) break;
+        if constexpr (kAttn) {
+          if (phase == 1) {
+            // the item's last O^T MMA, then O^T goes to the epilogue
+            if (!issue_pv()) {
+              ok = false;
+              break;
+            }
+            tc_commit(&ctl.o_full);
+            o_issued = 1;
+            last_opar = oi & 1u;
+            ++oi;
+          }
+        }
         tc_commit(&ctl.q_empty[qb]);
       }
       if (!ok) set_error(P, ctl, 1u);
@@ -778,6 +962,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       volatile int no_abort = 0;
       if (issued)
         mbar_wait(&ctl.acc_full[last_ab], last_par, P.wait_limit_ns, &no_abort);
+      if (kAttn && o_issued) mbar_wait(&ctl.o_full, last_opar, P.wait_limit_ns, &no_abort);
     }
   } else if (warp == kSyncWarp) {
     // ------------------------------------------------------------ sync warp
@@ -906,7 +1091,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const MergeJob job = ctl.merge_job[ms];
       if (job.unit < 0) break;
-      if (!merge_unit(P, ctl, job, mbuf, mphase)) {
+      if (!merge_unit<kAttn>(P, ctl, job, mbuf, mphase)) {
         set_error(P, ctl, 1u);
         // no bulk copy may still be writing shared memory when the CTA exits
         volatile int no_abort = 0;
@@ -919,7 +1104,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    uint32_t it = 0, ai = 0;
+    uint32_t it = 0, ai = 0, oi = 0;
     for (;;) {
       const uint32_t slot = it % kItemSlots;
       const uint32_t par = (it / kItemSlots) & 1u;
@@ -931,10 +1116,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (d.p < 0) break;
       bool ok;
       if (d.phase == 0) {
-        ok = rowstats_item<kFull>(P, ctl, d, slot, ai);
+        ok = rowstats_item<kFull, kAttn>(P, ctl, d, slot, ai);
       } else {
         ok = warp_wait(&ctl.beta_full[slot], par, P.wait_limit_ns, &ctl.abort) &&
-             colstats_item<kFull>(P, ctl, d, slot, ai);
+             colstats_item<kFull, kAttn>(P, ctl, d, slot, ai, kbuf, oi);
       }
       if (!ok) {
         set_error(P, ctl, 1u);
@@ -957,27 +1142,58 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-}  // namespace
 
-cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
-                         const ScoreParams& p, int ctas, cudaStream_t stream) {
-  const bool full = plan.geo.n_rows == kMaxRows;
-  auto* fn = full ? score_kernel<true> : score_kernel<false>;
-  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(kDynSmem));
+// Window output, last step: O of unit u's window rows = the sum of its column items'
+// partials (fp32), written as bf16 in q_win's layout (row r of the unit at q_row0 + r).
+__global__ void __launch_bounds__(kHeadDim) attn_finish_kernel(const __grid_constant__ Geometry g,
+                                                               const float* o_part, uint16_t* o_win) {
+  wait_previous_kernel();   // the partials come from the score kernel launched before
+  const UnitInfo u = unit_info(g, blockIdx.x);
+  const int j = threadIdx.x;   // head dimension
+  for (int r = 0; r < g.n_rows; ++r) {
+    float acc = 0.f;
+    for (int s = 0; s < u.splits; ++s)
+      acc += __ldcs(o_part + ((u.item0 + s) * kMaxRows + r) * kHeadDim + j);
+    uint32_t w;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w) : "f"(0.f), "f"(acc));
+    o_win[(u.q_row0 + r) * kHeadDim + j] = static_cast<uint16_t>(w & 0xFFFFu);
+  }
+}
+
+template <bool kAttn>
+cudaError_t launch_score_variant(bool full, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                                 const CUtensorMap& tm_v, const ScoreParams& p, int ctas, cudaStream_t stream) {
+  auto* fn = full ? score_kernel<true, kAttn> : score_kernel<false, kAttn>;
+  constexpr size_t smem = Cfg<kAttn>::kDynSmem;
+  cudaError_t e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   // CTAs wait on each other's row statistics: all of them must be resident at once
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(ctas));
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kDynSmem;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeCooperative;
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fn, tm_q, tm_k, p);
+  return cudaLaunchKernelEx(&cfg, fn, tm_q, tm_k, tm_v, p);
+}
+
+}  // namespace
+
+cudaError_t launch_score(const kve_plan& plan, const CUtensorMap& tm_q, const CUtensorMap& tm_k,
+                         const CUtensorMap* tm_v, const ScoreParams& p, int ctas, cudaStream_t stream) {
+  const bool full = plan.geo.n_rows == kMaxRows;
+  if (!tm_v) return launch_score_variant<false>(full, tm_q, tm_k, tm_k, p, ctas, stream);
+  return launch_score_variant<true>(full, tm_q, tm_k, *tm_v, p, ctas, stream);
+}
+
+cudaError_t launch_attn_finish(const kve_plan& plan, const float* o_part, uint16_t* o_win,
+                               cudaStream_t stream) {
+  return launch_after_previous(attn_finish_kernel, dim3(static_cast<unsigned>(plan.geo.n_units)),
+                               dim3(kHeadDim), 0, stream, plan.geo, o_part, o_win);
 }
 
 }  // namespace kve

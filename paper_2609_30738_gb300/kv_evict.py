@@ -20,7 +20,8 @@ KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 # Names declared in include/kv_evict.h.
 EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_destroy",
            "kv_evict_plan_set_debug", "kv_evict_plan_set_kv_strides",
-           "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
+           "kv_evict_score", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
+           "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
            "kv_evict_select_profiles_workspace", "kv_evict_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
 
@@ -62,6 +63,8 @@ def _lib():
         lib.kv_evict_plan_set_debug.argtypes = [vp, ctypes.c_uint64, i32]
         lib.kv_evict_plan_set_kv_strides.argtypes = [vp, vp, vp]
         lib.kv_evict_score.argtypes = [vp] * 7
+        lib.kv_evict_score_attn.argtypes = [vp] * 10
+        lib.kv_evict_score_attn_workspace.argtypes = [vp, vp]
         lib.kv_evict_select.argtypes = [vp] * 11
         lib.kv_evict_select_noalloc.argtypes = [vp] * 10
         lib.kv_evict_select_profiles.argtypes = [vp, i32] + [vp] * 10
@@ -73,7 +76,8 @@ def _lib():
         lib.kv_evict_strerror.restype = ctypes.c_char_p
         for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_set_debug",
                      "kv_evict_plan_set_kv_strides",
-                     "kv_evict_score", "kv_evict_select", "kv_evict_select_noalloc",
+                     "kv_evict_score", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
+                     "kv_evict_select", "kv_evict_select_noalloc",
                      "kv_evict_select_profiles", "kv_evict_select_profiles_workspace", "kv_evict_gather",
                      "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
             getattr(lib, name).restype = ctypes.c_int
@@ -191,6 +195,20 @@ class Plan:
     def score(self, q_win, k, mu, sigma, ws, stream=None):
         _check(_lib().kv_evict_score(self._h, _ptr(q_win), _ptr(k), _ptr(mu), _ptr(sigma), _ptr(ws),
                                      _stream_ptr(stream)), "kv_evict_score")
+
+    def score_attn_workspace(self) -> int:
+        """Bytes of the second scratch buffer of score_attn."""
+        out = ctypes.c_size_t(0)
+        _check(_lib().kv_evict_score_attn_workspace(self._h, ctypes.byref(out)),
+               "kv_evict_score_attn_workspace")
+        return out.value
+
+    def score_attn(self, q_win, k, v, mu, sigma, o_win, ws, attn_ws, stream=None):
+        """kv_evict_score_attn: score plus the window rows' attention output o_win
+        (q_win's layout, bf16)."""
+        _check(_lib().kv_evict_score_attn(self._h, _ptr(q_win), _ptr(k), _ptr(v), _ptr(mu), _ptr(sigma),
+                                          _ptr(o_win), _ptr(ws), _ptr(attn_ws), _stream_ptr(stream)),
+               "kv_evict_score_attn")
 
     def select(self, mu, sigma, k, lambda1, lambda2, indices, ws, order=None, margins=None,
                stream=None):

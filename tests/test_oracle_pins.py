@@ -509,6 +509,67 @@ def test_bf16_decode():
 
 
 # --------------------------------------------------------------------------
+# The window rows' attention output (Section 3.2: the existing attention)
+
+
+def test_window_output_uniform_keys_closed_form():
+    """All keys equal: every visible key gets 1/(p+1), so O[r] is the mean of the
+    values at positions 0 .. p_r (prefix means by cumulative sums)."""
+    rng = np.random.default_rng(41)
+    L, W, G, d = 24, 5, 3, 8
+    k = np.tile(rng.standard_normal(d), (L, 1))
+    q = rng.standard_normal((G * W, d))
+    v = rng.standard_normal((L, d))
+    O_ = O.window_output(O.window_attention(q, k, L, W, G), v)
+    prefix_mean = np.cumsum(v, axis=0) / np.arange(1, L + 1)[:, None]
+    for g in range(G):
+        for w in range(W):
+            np.testing.assert_allclose(O_[g * W + w], prefix_mean[L - W + w], rtol=1e-12, atol=1e-14)
+
+
+def test_window_output_single_visible_key():
+    """A window row at position 0 sees only key 0: its output is v_0 exactly."""
+    rng = np.random.default_rng(42)
+    L = W = 6
+    q = rng.standard_normal((W, 4)) * 3
+    k = rng.standard_normal((L, 4))
+    v = rng.standard_normal((L, 4))
+    O_ = O.window_output(O.window_attention(q, k, L, W, 1), v)
+    np.testing.assert_array_equal(O_[0], v[0])
+
+
+def test_window_output_matches_scipy_softmax():
+    rng = np.random.default_rng(43)
+    L, W, G, d = 30, 4, 2, 8
+    q, k = _rand_unit(rng, L, W, G, d)
+    v = rng.standard_normal((L, d))
+    O_ = O.window_output(O.window_attention(q, k, L, W, G), v)
+    for r in range(G * W):
+        p = L - W + (r % W)
+        a = scipy.special.softmax(np.array([q[r] @ k[i] for i in range(p + 1)]) / math.sqrt(d))
+        np.testing.assert_allclose(O_[r], a @ v[:p + 1], rtol=1e-12, atol=1e-14)
+
+
+def test_planted_window_output_bugs_are_caught(monkeypatch):
+    """Values paired with the wrong keys (positions reversed), or attention without the
+    causal mask, fail the pins."""
+    orig = O.window_attention
+    monkeypatch.setattr(O, "window_output", lambda A, v: A[:, ::-1] @ v)
+    with pytest.raises(AssertionError):
+        test_window_output_matches_scipy_softmax()
+    monkeypatch.setattr(O, "window_output", lambda A, v: A @ v)
+
+    def unmasked(q, k, L, W, G):
+        lg = (q @ k.T) / math.sqrt(q.shape[1])
+        e = np.exp(lg - lg.max(axis=1, keepdims=True))
+        return e / e.sum(axis=1, keepdims=True)
+    monkeypatch.setattr(O, "window_attention", unmasked)
+    with pytest.raises(AssertionError):
+        test_window_output_single_visible_key()
+    monkeypatch.setattr(O, "window_attention", orig)
+
+
+# --------------------------------------------------------------------------
 # Eq. 6
 
 
