@@ -409,8 +409,8 @@ __device__ __forceinline__ bool colstats_item(const ScoreParams& P, ScoreCtl& ct
     // of squares, m2 = sum A'^2 - (sum A')^2 / n
     const bool two = kFull || n > 64;
     float S1 = 0.f, SS = 0.f;
-#pragma unroll 1
     uint8_t* pt = kAttn ? kbuf + (ai % kKStages) * kTileBytes : nullptr;
+#pragma unroll 1
     for (int h = 0; h < (two ? 2 : 1); ++h) {
       float sh, qh;
       colsums_half<kFull, kAttn>(P, ctl, nb4, taddr, 64 * h, n, rel, sh, qh, pt, tl);

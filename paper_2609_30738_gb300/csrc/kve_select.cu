@@ -418,8 +418,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
           const uint32_t d = kb[j] >> 20;
           if (d > bin) {
             const uint32_t e = atomicAdd(&sh.cnt, 1u);
-            cpos[e] = i;
-            ckey[e] = kb[j];
+            if (e < static_cast<uint32_t>(NT)) {   // always, unless the count check below fails
+              cpos[e] = i;
+              ckey[e] = kb[j];
+            }
           } else if (d == bin) {
             const uint32_t e = atomicAdd(&sh.ncand, 1u);
             if (e < kCandCap<NT>()) {
@@ -452,8 +454,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       const uint32_t k = cand_k[e];
       if (k > T) {
         const uint32_t n = atomicAdd(&sh.cnt, 1u);
-        cpos[n] = cand_p[e];
-        ckey[n] = k;
+        if (n < static_cast<uint32_t>(NT)) {
+          cpos[n] = cand_p[e];
+          ckey[n] = k;
+        }
       } else if (k == T) {
         const uint32_t q = atomicAdd(&sh.teq, 1u);
         if (q < kTieCap) ties[q] = cand_p[e];
@@ -473,8 +477,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
         if (i < Lc) {
           if (kb[j] > T) {
             const uint32_t n = atomicAdd(&sh.cnt, 1u);
-            cpos[n] = i;
-            ckey[n] = kb[j];
+            if (n < static_cast<uint32_t>(NT)) {
+              cpos[n] = i;
+              ckey[n] = kb[j];
+            }
           } else if (kb[j] == T) {
             const uint32_t e = atomicAdd(&sh.teq, 1u);
             if (e < kTieCap) ties[e] = i;
@@ -488,8 +494,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   const uint32_t n_eq = sh.teq;
   // Every path above leaves n_above = #{key > T} and n_eq = #{key == T} with
   // n_above + needT = C and needT <= n_eq, so that the ties below fill the pool to
-  // exactly C positions. Should that ever fail, the pool would hold unwritten slots:
-  // the unit is then reported through the error word and gets no selection.
+  // exactly C positions (the pool writes above are bounded by the pool's size all the
+  // same). Should that ever fail, the pool would hold unwritten slots: the unit is then
+  // reported through the error word and gets no selection.
   if (n_above + needT != static_cast<uint32_t>(C) || needT > n_eq || needT == 0u) {
     if (tid == 0 && P.err) atomicOr(P.err, kErrCheck);
     int32_t* out = P.indices + out_off + u.unit * B;
