@@ -137,7 +137,7 @@ def test_window_output_strided_values():
 def test_window_output_full_size_sampled_units():
     """The L = 32768 workload (256 units, 38 work items each): sampled units' window
     output against the oracle. Here the window-output pass folds a unit's 38 row
-    partials in batches of 8 (its smaller merge buffer) where the plain pass folds them
+    partials in batches of 16 (its smaller merge buffer) where the plain pass folds them
     in one batch of 40, so the normalisers, and with them mu and sigma, may differ from
     the plain pass in the last bits: they are compared within 1e-5 relative."""
     spec = WORKLOADS["mistral-32layer-L32768-B64"]
