@@ -20,6 +20,7 @@ cores.
 from __future__ import annotations
 
 import argparse
+import gc
 import hashlib
 import json
 import math
@@ -46,8 +47,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "83af739a090d029d0a7839aa92903226e0a6d222029369867ae43459a7a495f6",
-                 "bytes_per_launch": 2173382144 + 74817280}
+SCORE_TRAFFIC = {"source_sha256": "c32b9fd1786d1a7070289b782563a05d965848b2b760c257d86159843b46000b",
+                 "bytes_per_launch": 2174652928 + 74828800}
 
 
 def _score_source_sha():
@@ -363,6 +364,11 @@ def run_ours(args):
             step()
     stream.synchronize()
 
+    # no garbage collection while GPU work is being enqueued: a collection pause of the
+    # host thread (tens of ms with torch loaded) would leave the GPU idle inside a timed
+    # region; collected once here and re-enabled after the last timed region
+    gc.collect()
+    gc.disable()
     sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
         sampler.start()
@@ -439,17 +445,20 @@ def run_ours(args):
     # whole tensor.
     e2e = None
     if args.e2e_steps > 0:
-        e2e_s, h2d, d2h, chunks = 0.0, 0, 0, 1
+        e2e_s, h2d, d2h, chunks, steps_ms = 0.0, 0, 0, 1, []
         if batch is not None:
-            e2e_s, h2d, d2h, chunks = _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream, dev, world)
+            e2e_s, h2d, d2h, chunks, steps_ms = _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream,
+                                                     dev, world)
         elif world > 1:
             dist.barrier()                 # the one in _e2e, for a rank without requests
         e2e_s = _max_over_ranks(e2e_s, world, dev)
         job_tokens = tokens * world if scaling == "weak" else sum(full["seq_lens"])
         e2e = {"value": job_tokens / e2e_s, "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "layer_chunks": chunks,
+               "step_ms_min_max": [min(steps_ms), max(steps_ms)] if steps_ms else None,
                "v": "read in place from pinned host memory by the gather (kept rows only)"}
 
+    gc.enable()
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -551,22 +560,25 @@ def _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream, dev, world):
     stream.synchronize()
     if cplan.status(cws, stream) != K.KVE_OK:
         raise RuntimeError("device-side wait timed out in the end-to-end step")
-    a = torch.cuda.Event(enable_timing=True)
-    b = torch.cuda.Event(enable_timing=True)
+    # an event at every step boundary (each step's copies wait for the previous step, so
+    # consecutive events bracket one step): the mean over the steps is the measurement,
+    # the spread is reported beside it
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.e2e_steps + 1)]
     if world > 1:
         dist.barrier()
     copy_stream.wait_stream(stream)
-    a.record(copy_stream)
-    for _ in range(args.e2e_steps):
+    ev[0].record(copy_stream)
+    for i in range(args.e2e_steps):
         e2e_step()
-    b.record(stream)
+        ev[i + 1].record(stream)
     torch.cuda.synchronize()
     if cplan.status(cws, stream) != K.KVE_OK:
         raise RuntimeError("device-side wait timed out in the end-to-end step")
-    e2e_s = a.elapsed_time(b) / 1e3 / args.e2e_steps
+    e2e_s = ev[0].elapsed_time(ev[-1]) / 1e3 / args.e2e_steps
+    steps_ms = [ev[i].elapsed_time(ev[i + 1]) for i in range(args.e2e_steps)]
     h2d = sum(x.numel() * x.element_size() for x in (hq, hk)) + v_read
     d2h = sum(x.numel() * x.element_size() for x in (o_idx, o_k, o_v))
-    return e2e_s, h2d, d2h, chunks
+    return e2e_s, h2d, d2h, chunks, steps_ms
 
 
 def cpu_baseline_from_device(spec, batch, n_units):
