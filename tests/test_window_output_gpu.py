@@ -7,8 +7,9 @@ bf16 (8 significant bits: relative rounding error <= 2^-8), the product accumula
 fp32, and O is rounded to bf16 once (<= 2^-8 |O|); so
 |O - O_ref| <= 2^-8 sum_i A_ri |v_ij| + 2^-8 |O_ref| (the probabilities' own fp32 error,
 ~1e-5 relative, is far below), checked here at twice that plus 1e-6 absolute. mu and
-sigma must equal kv_evict_score's bit for bit (within 1e-5 relative at full size, see
-that test), and the selection made from them likewise.
+sigma meet the oracle tolerances of every parity test, and stay within 1e-5 relative of
+kv_evict_score's (the two calls may fold a unit's row partials in different batches, so
+the normalisers can round differently in the last bits).
 """
 
 import numpy as np
@@ -55,9 +56,15 @@ def _run_both(spec, batch, per_query_head=False, kt=None, vt=None, k_strides=Non
     return (plan, bufs), (plan2, bufs2), (q, k, v), o_win
 
 
-def _check_outputs(spec, batch, o_win, per_query_head=False, units=None):
-    """O of the listed units (r, layer, head) against the oracle; returns the worst
-    |O - O_ref| / bound."""
+def _close(a, b, rtol=1e-5):
+    """Elementwise |a - b| <= rtol |b| + 1e-30 (float tensors on the device)."""
+    a, b = a.double(), b.double()
+    return bool(((a - b).abs() <= rtol * b.abs() + 1e-30).all())
+
+
+def _check_outputs(spec, batch, o_win, per_query_head=False, units=None, bufs=None):
+    """O of the listed units (r, layer, head) against the oracle, and (bufs given) mu and
+    sigma of the same call; returns the worst |O - O_ref| / bound."""
     seq = batch["seq_lens"]
     W, Hq, Hkv = spec["window"], spec["num_q_heads"], spec["num_kv_heads"]
     G = Hq // Hkv
@@ -77,6 +84,12 @@ def _check_outputs(spec, batch, o_win, per_query_head=False, units=None):
         A = O.window_attention(O.bf16_bits_to_f64(qb), O.bf16_bits_to_f64(kb), L, W, ug)
         o_ref = O.window_output(A, vf)
         o_gpu = ow[layer, r, h * ug:(h + 1) * ug].reshape(ug * W, -1)
+        if bufs is not None:
+            mu_ref = O.mean_attention(A)
+            sg_ref = O.dispersion(A, mu_ref)
+            o0 = spec["num_layers"] * uheads * off + (layer * uheads + h) * L
+            PT.check_mu_sigma(bufs.mu[o0:o0 + L].cpu().numpy(), bufs.sigma[o0:o0 + L].cpu().numpy(),
+                              mu_ref, sg_ref, f"unit (r={r}, l={layer}, h={h})")
         bound = O_REL * (A @ np.abs(vf)) + O_REL * np.abs(o_ref) + 1e-6
         err = np.abs(o_gpu - o_ref)
         bad = np.argwhere(~(err <= bound))
@@ -88,23 +101,42 @@ def _check_outputs(spec, batch, o_win, per_query_head=False, units=None):
 
 @pytest.mark.parametrize("case", ["L2048", "ragged"])
 def test_window_output_every_unit(case):
-    """Every unit's window output against the oracle; mu, sigma and the selection made
-    from them equal the plain score pass bit for bit."""
-    from paper_2609_30738_gb300 import kv_evict as K
+    """Every unit's window output, mu and sigma against the oracle; mu and sigma within
+    1e-5 relative of the plain score pass."""
     if case == "L2048":
         spec = WORKLOADS["mistral-1layer-L2048"]
     else:
         spec = scaled(WORKLOADS["mistral-1layer-L2048"], num_layers=2, budget=16, seq_lens=[300, 777, 1500, 513])
     batch = synth.make_batch(spec, seed=71)
     (plan, bufs), (plan2, bufs2), (q, k, v), o_win = _run_both(spec, batch)
-    assert torch.equal(bufs.mu, bufs2.mu) and torch.equal(bufs.sigma, bufs2.sigma)
-    lam = lambda_arrays(spec, K.profile)
-    for pl, bf in ((plan, bufs), (plan2, bufs2)):
-        pl.select(bf.mu, bf.sigma, k, lam[0], lam[1], bf.indices, bf.ws, bf.order, bf.margins)
-    assert plan2.status(bufs2.ws) == K.KVE_OK
-    assert torch.equal(bufs.indices, bufs2.indices) and torch.equal(bufs.margins, bufs2.margins)
-    worst = _check_outputs(spec, batch, o_win)
+    assert _close(bufs2.mu, bufs.mu) and _close(bufs2.sigma, bufs.sigma)
+    worst = _check_outputs(spec, batch, o_win, bufs=bufs2)
     print(f"window output, worst |O - O_ref| / bound = {worst:.3f}")
+
+
+def test_window_output_logit_jump():
+    """Keys whose logits exceed everything earlier in their work item by far (planted:
+    k = c q_r for one window row r, logit about 200 in natural units, i.e. 2^288 times
+    the rest): the rows' maxima and normalisers jump in the middle of an item. O, mu and
+    sigma against the oracle on every unit."""
+    spec = scaled(WORKLOADS["mistral-1layer-L2048"], budget=16, seq_lens=[2048, 1536])
+    batch = synth.make_batch(spec, seed=75)
+    q, k = batch["q_win"], batch["k"]
+    W, G, d = spec["window"], spec["num_q_heads"] // spec["num_kv_heads"], spec["head_dim"]
+    off = 0
+    for r, L in enumerate(spec["seq_lens"]):
+        for h in range(spec["num_kv_heads"]):
+            for j, pos in enumerate((128 * 5 + 7, 128 * 11 + 3)):
+                if pos >= L - W:
+                    continue
+                qr = q[0, r, h * G + (j % G), (3 * j + h) % W].double()
+                c = 200.0 * d ** 0.5 / float((qr * qr).sum())
+                k[0, h, off + pos] = (c * qr).to(k.dtype)
+        off += L
+    (_, bufs), (_, bufs2), _, o_win = _run_both(spec, batch)
+    worst = _check_outputs(spec, batch, o_win, bufs=bufs2)
+    assert _close(bufs2.mu, bufs.mu, 1e-4) and _close(bufs2.sigma, bufs.sigma, 1e-4)
+    print(f"logit jump, worst |O - O_ref| / bound = {worst:.3f}")
 
 
 def test_window_output_short_rows_and_per_query_head():
@@ -113,13 +145,13 @@ def test_window_output_short_rows_and_per_query_head():
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], window=8, budget=16, seq_lens=[1000, 129])
     batch = synth.make_batch(spec, seed=72)
     (_, bufs), (_, bufs2), _, o_win = _run_both(spec, batch)
-    assert torch.equal(bufs.mu, bufs2.mu) and torch.equal(bufs.sigma, bufs2.sigma)
-    _check_outputs(spec, batch, o_win)
+    assert _close(bufs2.mu, bufs.mu) and _close(bufs2.sigma, bufs.sigma)
+    _check_outputs(spec, batch, o_win, bufs=bufs2)
     spec = scaled(WORKLOADS["mistral-1layer-L2048"], budget=16, seq_lens=[900, 300])
     batch = synth.make_batch(spec, seed=73)
     (_, bufs), (_, bufs2), _, o_win = _run_both(spec, batch, per_query_head=True)
-    assert torch.equal(bufs.mu, bufs2.mu) and torch.equal(bufs.sigma, bufs2.sigma)
-    _check_outputs(spec, batch, o_win, per_query_head=True)
+    assert _close(bufs2.mu, bufs.mu) and _close(bufs2.sigma, bufs.sigma)
+    _check_outputs(spec, batch, o_win, per_query_head=True, bufs=bufs2)
 
 
 def test_window_output_strided_values():
@@ -136,16 +168,12 @@ def test_window_output_strided_values():
 
 def test_window_output_full_size_sampled_units():
     """The L = 32768 workload (256 units, 38 work items each): sampled units' window
-    output against the oracle. Here the window-output pass folds a unit's 38 row
-    partials in batches of 16 (its smaller merge buffer) where the plain pass folds them
-    in one batch of 40, so the normalisers, and with them mu and sigma, may differ from
-    the plain pass in the last bits: they are compared within 1e-5 relative."""
+    output, mu and sigma against the oracle; mu and sigma within 1e-5 relative of the
+    plain score pass everywhere."""
     spec = WORKLOADS["mistral-32layer-L32768-B64"]
     batch = synth.make_batch(spec, seed=2609, device=DEV)
     (_, bufs), (_, bufs2), _, o_win = _run_both(spec, batch)
-    for a, b in ((bufs.mu, bufs2.mu), (bufs.sigma, bufs2.sigma)):
-        rel = ((a.double() - b.double()).abs() / a.double().abs().clamp_min(1e-30)).max().item()
-        assert rel <= 1e-5, rel
+    assert _close(bufs2.mu, bufs.mu) and _close(bufs2.sigma, bufs.sigma)
     units = [(0, 0, 0), (0, 13, 5), (0, 31, 7)]
-    worst = _check_outputs(spec, batch, o_win, units=units)
+    worst = _check_outputs(spec, batch, o_win, units=units, bufs=bufs2)
     print(f"full size window output, worst |O - O_ref| / bound = {worst:.3f}")
