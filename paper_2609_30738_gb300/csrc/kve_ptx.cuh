@@ -79,6 +79,17 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64
   }
 }
 
+// Two waits whose first polls are issued together, so that their latencies overlap when
+// both barriers are ready (the common case on a critical path); otherwise the bounded
+// waits above, one after the other.
+__device__ __forceinline__ bool mbar_wait2(uint64_t* bar_a, uint32_t parity_a, uint64_t* bar_b,
+                                           uint32_t parity_b, uint64_t limit_ns, volatile int* abort) {
+  const bool a = mbar_try_wait(bar_a, parity_a);
+  const bool b = mbar_try_wait(bar_b, parity_b);
+  if (a && b) return true;
+  return (a || mbar_wait(bar_a, parity_a, limit_ns, abort)) && (b || mbar_wait(bar_b, parity_b, limit_ns, abort));
+}
+
 // ---------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int32_t x,

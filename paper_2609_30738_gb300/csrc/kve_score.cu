@@ -907,10 +907,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int t = 0; t < ntiles; ++t) {
           const uint32_t ks = ki % kKStages;
           const uint32_t ab = ai % kAccBufs;
-          if (!mbar_wait(&ctl.k_full[ks], (ki / kKStages) & 1u, P.wait_limit_ns,
-                         &ctl.abort) ||
-              !mbar_wait(&ctl.acc_empty[ab], ((ai / kAccBufs) & 1u) ^ 1u,
-                         P.wait_limit_ns, &ctl.abort)) {
+          if (!mbar_wait2(&ctl.k_full[ks], (ki / kKStages) & 1u, &ctl.acc_empty[ab],
+                          ((ai / kAccBufs) & 1u) ^ 1u, P.wait_limit_ns, &ctl.abort)) {
             ok = false;
             break;
           }
