@@ -47,8 +47,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "c32b9fd1786d1a7070289b782563a05d965848b2b760c257d86159843b46000b",
-                 "bytes_per_launch": 2174652928 + 74828800}
+SCORE_TRAFFIC = {"source_sha256": "27a8cccde14384233815968591af65ffb1f9b01ff25a7eb4ecabba3d581a2184",
+                 "bytes_per_launch": 2180194048 + 74918400}
 
 
 def _score_source_sha():
@@ -456,6 +456,7 @@ def run_ours(args):
         e2e = {"value": job_tokens / e2e_s, "unit": "prefix tok/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "layer_chunks": chunks,
                "step_ms_min_max": [min(steps_ms), max(steps_ms)] if steps_ms else None,
+               "step_ms_median": sorted(steps_ms)[len(steps_ms) // 2] if steps_ms else None,
                "v": "read in place from pinned host memory by the gather (kept rows only)"}
 
     gc.enable()
@@ -615,7 +616,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=BENCH_WORKLOADS, default=WORKLOAD)
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--e2e-chunks", type=int, default=8,
                     help="layer chunks of the end-to-end step (copy of chunk c+1 beside compute of c)")
     ap.add_argument("--cpu-units", type=int, default=128)
