@@ -28,6 +28,9 @@ namespace kve {
 namespace {
 
 constexpr int kChunks = kHeadDim / 8;   // 16-byte chunks of a key row
+constexpr int kRowChunks = kChunks + 1; // staged row pitch (272 bytes): the 8 rows of an
+                                        // mma fragment load fall on distinct banks
+constexpr int kRowWords = 4 * kRowChunks;
 constexpr int kBins = 4096;             // radix digits of the first two passes
 constexpr int kPoolRun = 7;             // consecutive pooled outputs per run (odd: the
                                         // runs of a warp start on distinct banks)
@@ -47,6 +50,18 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return d;
 }
 
+// 1/sqrt(x) for x > 0: the hardware estimate refined by one Newton-Raphson step,
+// y <- y + y (1 - x y^2) / 2 (within about an ulp); x below 2^-64 is scaled by 2^64
+// first, so that the estimate never sees a subnormal argument.
+__device__ __forceinline__ float inv_sqrt(float x) {
+  const bool tiny = x < 0x1p-64f;
+  const float xs = tiny ? x * 0x1p64f : x;
+  const float y = rsqrtf(xs);
+  const float e = fmaf(-xs * y, y, 1.0f);
+  const float r = fmaf(0.5f * y, e, y);
+  return tiny ? r * 0x1p32f : r;
+}
+
 __device__ __forceinline__ float unord_key(uint32_t k) {
   const uint32_t u = (k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k;
   return __uint_as_float(u);
@@ -63,7 +78,7 @@ struct SelSmall {
 // finer-digit histogram in the `big` region
 template <int NT>
 __host__ __device__ constexpr uint32_t kCandCap() {
-  return static_cast<uint32_t>((kChunks * NT * sizeof(uint4) - kBins * sizeof(uint32_t)) /
+  return static_cast<uint32_t>((kRowChunks * NT * sizeof(uint4) - kBins * sizeof(uint32_t)) /
                                (sizeof(uint32_t) + sizeof(int32_t)));
 }
 
@@ -115,7 +130,7 @@ struct OneProfile {
 };
 
 template <int NT, class Prof>
-__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams P,
+__global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __grid_constant__ SelectParams P,
                                                     const __grid_constant__ Prof prof) {
   __shared__ SelSmall<NT> sh;
   extern __shared__ __align__(16) uint8_t dyn[];
@@ -149,10 +164,10 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   // turn the pooling tiles, the radix histogram and tie list, the threshold bin's
   // (key, position) pairs, and the staged candidate keys
   uint8_t* big = dyn;
-  uint4* krow = reinterpret_cast<uint4*>(big);                                  // [NT][kChunks]
+  uint4* krow = reinterpret_cast<uint4*>(big);                                  // [NT][kRowChunks]
   uint32_t* hist12 = reinterpret_cast<uint32_t*>(big);                          // [kBins] later passes
   float* tmu = reinterpret_cast<float*>(big);                                   // pooling tiles
-  int32_t* cpos = reinterpret_cast<int32_t*>(big + kChunks * NT * sizeof(uint4));   // pool positions
+  int32_t* cpos = reinterpret_cast<int32_t*>(big + kRowChunks * NT * sizeof(uint4));   // pool positions
   uint32_t* ckey = reinterpret_cast<uint32_t*>(cpos + NT);                      // and their keys
   int32_t* spos = reinterpret_cast<int32_t*>(ckey + NT);                        // sorted pool (or the
   uint32_t* skey = reinterpret_cast<uint32_t*>(spos + NT);                      // admitted positions)
@@ -577,19 +592,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
 #pragma unroll
     for (int q = 0; q < kRows; ++q) {
       const int r = (q * (NT / 32) + warp) * 2 + (lane >> 4);
-      if (r < C) krow[r * kChunks + (lane & 15)] = xr[q];
-      const uint32_t w4[4] = {xr[q].x, xr[q].y, xr[q].z, xr[q].w};
-      float ss = 0.f;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float lo = __uint_as_float(w4[e] << 16);
-        const float hi = __uint_as_float(w4[e] & 0xFFFF0000u);
-        ss = fmaf(lo, lo, ss);
-        ss = fmaf(hi, hi, ss);
-      }
-#pragma unroll
-      for (int o = 8; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-      if (r < C && (lane & 15) == 0) inv[r] = ss > 0.f ? __fdiv_rn(1.0f, sqrtf(ss)) : 0.f;
+      if (r < C) krow[r * kRowChunks + (lane & 15)] = xr[q];
     }
   }
   __syncthreads();
@@ -606,21 +609,42 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   bool active = slot < C;
   float corr = 0.f;
   const float my_st = active ? __fdiv_rn(unord_key(pkey[slot]), smax) : 0.f;
-  const float my_inv = active ? inv[slot] : 0.f;
+  // the candidate's inverse norm, from its own staged row (the admitted key's comes
+  // from inv[] after the first barrier of the loop below)
+  float my_inv = 0.f;
+  if (active) {
+    const uint4* row = krow + slot * kRowChunks;
+    float ss0 = 0.f, ss1 = 0.f;
+#pragma unroll 4
+    for (int c = 0; c < kChunks; ++c) {
+      const uint4 w = row[c];
+      const uint32_t w4[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float lo = __uint_as_float(w4[e] << 16);
+        const float hi = __uint_as_float(w4[e] & 0xFFFF0000u);
+        ss0 = fmaf(lo, lo, ss0);
+        ss1 = fmaf(hi, hi, ss1);
+      }
+    }
+    const float ss = ss0 + ss1;
+    my_inv = ss > 0.f ? inv_sqrt(ss) : 0.f;
+    inv[slot] = my_inv;
+  }
   const uint32_t my_tie = !active ? 0xFFFFFFFFu
                                   : (packed ? (static_cast<uint32_t>(ppos[slot]) << 9) | static_cast<uint32_t>(slot)
                                             : static_cast<uint32_t>(slot));
-  const uint32_t* kw = reinterpret_cast<const uint32_t*>(krow);   // 64 words per row
+  const uint32_t* kw = reinterpret_cast<const uint32_t*>(krow);   // 4 * kRowChunks words per row
   uint32_t afr[2][8][4];
 #pragma unroll
   for (int m = 0; m < 2; ++m) {
     const int r0 = warp * 32 + 16 * m + g, r1 = r0 + 8;
 #pragma unroll
     for (int s8 = 0; s8 < 8; ++s8) {
-      afr[m][s8][0] = r0 < C ? kw[r0 * 64 + 8 * s8 + tq] : 0u;
-      afr[m][s8][1] = r1 < C ? kw[r1 * 64 + 8 * s8 + tq] : 0u;
-      afr[m][s8][2] = r0 < C ? kw[r0 * 64 + 8 * s8 + tq + 4] : 0u;
-      afr[m][s8][3] = r1 < C ? kw[r1 * 64 + 8 * s8 + tq + 4] : 0u;
+      afr[m][s8][0] = r0 < C ? kw[r0 * kRowWords + 8 * s8 + tq] : 0u;
+      afr[m][s8][1] = r1 < C ? kw[r1 * kRowWords + 8 * s8 + tq] : 0u;
+      afr[m][s8][2] = r0 < C ? kw[r0 * kRowWords + 8 * s8 + tq + 4] : 0u;
+      afr[m][s8][3] = r1 < C ? kw[r1 * kRowWords + 8 * s8 + tq + 4] : 0u;
     }
   }
   int32_t* order = P.order ? P.order + out_off + u.unit * B : nullptr;
@@ -671,8 +695,8 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
     uint32_t bf[8][2];
 #pragma unroll
     for (int s8 = 0; s8 < 8; ++s8) {
-      bf[s8][0] = kw[js * 64 + 8 * s8 + tq];
-      bf[s8][1] = kw[js * 64 + 8 * s8 + tq + 4];
+      bf[s8][0] = kw[js * kRowWords + 8 * s8 + tq];
+      bf[s8][1] = kw[js * kRowWords + 8 * s8 + tq + 4];
     }
 #pragma unroll
     for (int s8 = 0; s8 < 8; ++s8) {
@@ -721,12 +745,12 @@ template <int NT>
 constexpr size_t select_smem() {
   // candidate keys (also reused for the pooling tiles, the histograms, the threshold
   // bin's keys and the tie list) + 5 arrays + the first-digit histogram
-  return kChunks * NT * sizeof(uint4) + 5 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
+  return kRowChunks * NT * sizeof(uint4) + 5 * NT * sizeof(int32_t) + kBins * sizeof(uint32_t);
 }
-static_assert(kChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histogram fits");
-static_assert(kChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
+static_assert(kRowChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "histogram fits");
+static_assert(kRowChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
               "pool tiles fit");
-static_assert(kChunks * 256 * sizeof(uint4) >= kTieCap * sizeof(int32_t), "tie list fits");
+static_assert(kRowChunks * 256 * sizeof(uint4) >= kTieCap * sizeof(int32_t), "tie list fits");
 // both parameter blocks of a multi-profile launch fit the 32764-byte kernel
 // parameter space
 static_assert(sizeof(SelectParams) + sizeof(ProfileTable) + 64 <= 32764, "profile table fits");
