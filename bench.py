@@ -380,12 +380,13 @@ def run_ours(args):
     if sampler:
         sampler.mark("t0")
     t0.record(stream)
-    # no event between the launches: select and gather start as programmatic dependents
-    # of the kernel before them, which an event record in between would prevent
+    # no event between the launches: the selection (with the compact cache) starts as a
+    # programmatic dependent of the score kernel, which an event record in between would
+    # prevent
     for i in range(args.steps if batch is not None else 0):
         plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws, stream)
-        plan.select(bufs.mu, bufs.sigma, k, lam1, lam2, bufs.indices, bufs.ws, None, None, stream)
-        plan.gather(k, v, bufs.indices, bufs.k_out, bufs.v_out, stream)
+        plan.select_gather(bufs.mu, bufs.sigma, k, v, lam1, lam2, bufs.indices, bufs.k_out, bufs.v_out,
+                           bufs.ws, None, None, stream)
     t1.record(stream)
     torch.cuda.synchronize()
     if sampler:
@@ -395,7 +396,7 @@ def run_ours(args):
     elapsed = t0.elapsed_time(t1) / 1e3
     # the dominant kernel's launch duration for the roofline: the same number of steps
     # right after the timed region, an event pair around each score launch on the bench
-    # stream (select and gather still run between them)
+    # stream (the selection still runs between them)
     score_s = 0.0
     if batch is not None:
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -404,8 +405,8 @@ def run_ours(args):
             ev[i][0].record(stream)
             plan.score(q, k, bufs.mu, bufs.sigma, bufs.ws, stream)
             ev[i][1].record(stream)
-            plan.select(bufs.mu, bufs.sigma, k, lam1, lam2, bufs.indices, bufs.ws, None, None, stream)
-            plan.gather(k, v, bufs.indices, bufs.k_out, bufs.v_out, stream)
+            plan.select_gather(bufs.mu, bufs.sigma, k, v, lam1, lam2, bufs.indices, bufs.k_out,
+                               bufs.v_out, bufs.ws, None, None, stream)
         torch.cuda.synchronize()
         score_s = sum(a.elapsed_time(b) for a, b in ev) / 1e3 / args.steps
     clocks = sampler.stop() if sampler else None
@@ -440,9 +441,9 @@ def run_ours(args):
     # A one-request call is evicted in chunks of layers, one plan per chunk: the copy
     # stream brings in chunk c + 1 while the compute stream scores, selects and
     # gathers chunk c (every array is layer-major for one request, so a chunk is a
-    # contiguous view). V stays in pinned host memory: the gather reads the kept rows
-    # in place, so min(B_l, L_r - W) + W rows per unit cross the host link, not the
-    # whole tensor.
+    # contiguous view). V stays in pinned host memory: the selection's compact-cache
+    # write reads the kept rows in place, so min(B_l, L_r - W) + W rows per unit cross
+    # the host link, not the whole tensor.
     e2e = None
     if args.e2e_steps > 0:
         e2e_s, h2d, d2h, chunks, steps_ms = 0.0, 0, 0, 1, []
@@ -457,7 +458,7 @@ def run_ours(args):
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_s * 1e3, "layer_chunks": chunks,
                "step_ms_min_max": [min(steps_ms), max(steps_ms)] if steps_ms else None,
                "step_ms_median": sorted(steps_ms)[len(steps_ms) // 2] if steps_ms else None,
-               "v": "read in place from pinned host memory by the gather (kept rows only)"}
+               "v": "read in place from pinned host memory by the compact-cache write (kept rows only)"}
 
     gc.enable()
     if rank != 0:
@@ -497,7 +498,7 @@ def run_ours(args):
                          "peak_source": peak_kind, "kernel": "kve score_kernel",
                          "algorithmic_bytes_per_launch": k_read,
                          "secondary_bytes_per_launch": secondary},
-            "gpu_launches": 3 * args.steps,
+            "gpu_launches": 2 * args.steps,
             "clocks": clocks, "cpu_baseline": cpu, "e2e": e2e, "window_output": window}
     print(json.dumps(line), flush=True)
     if world > 1:
@@ -548,9 +549,8 @@ def _e2e(args, spec, batch, plan, bufs, lam1, lam2, stream, dev, world):
             ls = slice(c * Lc, (c + 1) * Lc)
             stream.wait_event(arrived[c])
             cplan.score(dq[ls], dk[ls], mu_c[c], sg_c[c], cws, stream)
-            cplan.select(mu_c[c], sg_c[c], dk[ls], lam1[ls], lam2[ls], idx_c[c], cws, None, None,
-                         stream)
-            cplan.gather(dk[ls], hv[ls], idx_c[c], ko_c[c], vo_c[c], stream)
+            cplan.select_gather(mu_c[c], sg_c[c], dk[ls], hv[ls], lam1[ls], lam2[ls], idx_c[c], ko_c[c],
+                                vo_c[c], cws, None, None, stream)
         with torch.cuda.stream(stream):
             o_idx.copy_(bufs.indices, non_blocking=True)
             o_k.copy_(bufs.k_out, non_blocking=True)

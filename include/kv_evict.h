@@ -191,6 +191,23 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu,
                            int32_t* indices, int32_t* order, float* margins,
                            void* ws, void* stream);
 
+/* Steps 3 and 4 in one launch: exactly what kv_evict_select followed by
+ * kv_evict_gather writes (indices, order, margins, k_out, v_out; the same arguments
+ * and the same layouts), with the compact cache written by the selection's own CTA
+ * for each unit: the kept key rows come from the copy the selection stages for its
+ * cosines (Eq. 4), so only the values and the window rows are read again. v may be
+ * page-locked host memory as for kv_evict_gather (and k as well). Returns KVE_EINVAL
+ * on the conditions of either call. For a plan whose selection runs over every
+ * candidate (candidate_factor 0 beyond 512 prefix tokens) the two steps stay two
+ * launches. */
+kve_status kv_evict_select_gather(const kve_plan* plan, const float* mu,
+                                  const float* sigma, const uint16_t* k,
+                                  const uint16_t* v, const float* lambda1,
+                                  const float* lambda2, int32_t* indices,
+                                  int32_t* order, float* margins,
+                                  uint16_t* k_out, uint16_t* v_out, void* ws,
+                                  void* stream);
+
 /* Step 3 for n_profiles profiles of the layer-wise coefficients in one pass over
  * the units (Section 3.3 searches over profiles and re-selects for each; mu and
  * sigma do not depend on the coefficients, so one kv_evict_score serves them all).

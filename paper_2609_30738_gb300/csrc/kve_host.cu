@@ -379,6 +379,17 @@ int32_t profiles_per_launch(const kve_plan* plan) {
   return kve::kProfileLambdas / (2 * plan->geo.num_layers);
 }
 
+// Sources of the compact cache may be pinned host memory (read in place under unified
+// addressing); host memory the CUDA runtime does not know is refused.
+bool readable_source(const void* src) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, src) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type != cudaMemoryTypeUnregistered;
+}
+
 }  // namespace
 
 extern "C" {
@@ -398,6 +409,33 @@ kve_status kv_evict_select(const kve_plan* plan, const float* mu, const float* s
     return kve::launch_select_all(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK
                                                                                               : KVE_ECUDA;
   }
+  return kve::launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
+}
+
+kve_status kv_evict_select_gather(const kve_plan* plan, const float* mu, const float* sigma, const uint16_t* k,
+                                  const uint16_t* v, const float* lambda1, const float* lambda2,
+                                  int32_t* indices, int32_t* order, float* margins, uint16_t* k_out,
+                                  uint16_t* v_out, void* ws, void* stream) {
+  if (!plan || !mu || !sigma || !k || !v || !lambda1 || !lambda2 || !indices || !k_out || !v_out || !ws)
+    return KVE_EINVAL;
+  if (!aligned(k, 16) || !aligned(v, 16) || !aligned(k_out, 16) || !aligned(v_out, 16) || !aligned(mu, 16) ||
+      !aligned(sigma, 16) || !aligned(ws, 256))
+    return KVE_EINVAL;
+  if (!readable_source(k) || !readable_source(v)) return KVE_EINVAL;
+  if (plan->select_all) {
+    // the every-candidate selector keeps its own launch; the gather follows it
+    const kve_status s = kv_evict_select(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, ws,
+                                         stream);
+    return s != KVE_OK ? s : kv_evict_gather(plan, k, v, indices, k_out, v_out, stream);
+  }
+  kve::SelectParams p;
+  const kve_status s = select_params(plan, mu, sigma, k, lambda1, lambda2, indices, order, margins, &p);
+  if (s != KVE_OK) return s;
+  p.keys = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.keys);
+  p.err = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + plan->ws.hdr);
+  p.v = v;
+  p.k_out = k_out;
+  p.v_out = v_out;
   return kve::launch_select(*plan, p, static_cast<cudaStream_t>(stream)) == cudaSuccess ? KVE_OK : KVE_ECUDA;
 }
 
@@ -453,16 +491,7 @@ kve_status kv_evict_gather(const kve_plan* plan, const uint16_t* k, const uint16
                            uint16_t* k_out, uint16_t* v_out, void* stream) {
   if (!plan || !k || !v || !indices || !k_out || !v_out) return KVE_EINVAL;
   if (!aligned(k, 16) || !aligned(v, 16) || !aligned(k_out, 16) || !aligned(v_out, 16)) return KVE_EINVAL;
-  // k and v may be pinned host memory (read in place under unified addressing);
-  // host memory the CUDA runtime does not know is refused
-  for (const void* src : {static_cast<const void*>(k), static_cast<const void*>(v)}) {
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, src) != cudaSuccess) {
-      cudaGetLastError();
-      return KVE_EINVAL;
-    }
-    if (at.type == cudaMemoryTypeUnregistered) return KVE_EINVAL;
-  }
+  if (!readable_source(k) || !readable_source(v)) return KVE_EINVAL;
   kve::GatherParams p;
   std::memset(&p, 0, sizeof(p));
   p.g = plan->geo;

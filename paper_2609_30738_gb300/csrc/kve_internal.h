@@ -150,6 +150,9 @@ struct SelectParams {
                              // hold exactly C positions, or a pool position outside the unit
   float* corr;               // workspace scratch of the every-candidate selector (or null):
                              // float2 (corr, 1/|k|) per prefix token of every unit
+  const uint16_t* v;         // with k_out and v_out: the selection also writes the compact
+  uint16_t* k_out;           // cache of step 4 (as the gather kernel does), or null
+  uint16_t* v_out;
   float lambda1[kMaxLayers];
   float lambda2[kMaxLayers];
   int32_t layer_budget[kMaxLayers];   // B_l <= budget kept candidates of layer l

@@ -123,6 +123,55 @@ __device__ __forceinline__ uint32_t block_excl_suffix(uint32_t x, SelSmall<NT>& 
   return incl - x + after;
 }
 
+// Step 4 in the selection's CTA (P.k_out set): unit u's compact cache [B + W][d] as the
+// gather kernel writes it. Rows r < nvalid are the kept candidates in ascending position
+// (rpos[r]; their key rows are still staged in shared memory, row rslot[r]); rows
+// m .. m+W-1 are the window tokens Lc .. L-1; every other row is zero. A half-warp
+// copies a 256-byte row with 16-byte accesses; all loads of a batch are in flight before
+// its first store. The copy is bit-exact.
+template <int NT>
+__device__ __forceinline__ void write_compact_cache(const SelectParams& P, const UnitInfo& u, int Lc, int m,
+                                                    int nvalid, const int32_t* rpos, const int32_t* rslot,
+                                                    const uint4* krow) {
+  constexpr int kRowsPerPass = NT / 16;
+  constexpr int kPasses = 8;
+  const int W = P.g.window;
+  const int rows = P.budget + W;
+  const int half = threadIdx.x >> 4, lane16 = threadIdx.x & 15;
+  const uint16_t* ksrc = P.k + u.k_off;
+  const uint16_t* vsrc = P.v + u.v_off;
+  uint4* kdst = reinterpret_cast<uint4*>(P.k_out + static_cast<int64_t>(u.unit) * rows * kHeadDim);
+  uint4* vdst = reinterpret_cast<uint4*>(P.v_out + static_cast<int64_t>(u.unit) * rows * kHeadDim);
+  for (int r0 = 0; r0 < rows; r0 += kPasses * kRowsPerPass) {
+    uint4 kv[kPasses], vv[kPasses];
+#pragma unroll
+    for (int p = 0; p < kPasses; ++p) {
+      const int r = r0 + p * kRowsPerPass + half;
+      kv[p] = make_uint4(0, 0, 0, 0);
+      vv[p] = make_uint4(0, 0, 0, 0);
+      if (r < nvalid) {
+        const int s = rpos[r];
+        if (s >= 0 && s < Lc) {                      // never read outside the unit
+          kv[p] = krow[rslot[r] * kRowChunks + lane16];
+          vv[p] = __ldcs(reinterpret_cast<const uint4*>(vsrc + s * P.g.v_st) + lane16);
+        }
+      } else if (r >= m && r < m + W) {
+        const int s = Lc + (r - m);
+        kv[p] = __ldcs(reinterpret_cast<const uint4*>(ksrc + s * P.g.k_st) + lane16);
+        vv[p] = __ldcs(reinterpret_cast<const uint4*>(vsrc + s * P.g.v_st) + lane16);
+      }
+    }
+#pragma unroll
+    for (int p = 0; p < kPasses; ++p) {
+      const int r = r0 + p * kRowsPerPass + half;
+      if (r < rows) {
+        kdst[static_cast<int64_t>(r) * (kHeadDim / 8) + lane16] = kv[p];
+        vdst[static_cast<int64_t>(r) * (kHeadDim / 8) + lane16] = vv[p];
+      }
+    }
+  }
+}
+
 // The coefficients of one selection: those of SelectParams (kMulti = false), or
 // profile first + blockIdx.y of a table (kMulti = true).
 struct OneProfile {
@@ -520,6 +569,7 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
       for (int r = tid; r < B; r += NT) P.order[out_off + u.unit * B + r] = -1;
     if (P.margins)
       for (int r = tid; r < B; r += NT) P.margins[out_off + u.unit * B + r] = 0.f;
+    if (P.k_out) write_compact_cache<NT>(P, u, Lc, nsel, 0, nullptr, nullptr, nullptr);
     return;
   }
   if (n_eq <= kTieCap) {
@@ -649,8 +699,10 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
   }
   int32_t* order = P.order ? P.order + out_off + u.unit * B : nullptr;
   float* margins = P.margins ? P.margins + out_off + u.unit * B : nullptr;
-  // admitted positions in admission order (the pool's other pair of arrays is free)
+  // admitted positions in admission order (the pool's other pair of arrays is free),
+  // and their slots when the compact cache is written here
   int32_t* adm = packed ? spos : cpos;
+  int32_t* adm_slot = reinterpret_cast<int32_t*>(packed ? skey : ckey);
   for (int t = 0; t < nsel; ++t) {
     const uint32_t key = active ? ord_key(fmaf(lambda2, corr, my_st)) : 0u;
     const uint32_t wmax = __reduce_max_sync(0xffffffffu, key);
@@ -679,6 +731,7 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
     if (tid == 0) {
       const int pos = packed ? static_cast<int>(btie >> 9) : ppos[js];
       adm[t] = pos;
+      adm_slot[t] = js;
       if (order) order[t] = pos;
       if (margins) margins[t] = sec ? unord_key(best) - unord_key(sec) : INFINITY;
     }
@@ -728,17 +781,29 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
   // 6. admitted positions in ascending order (rank among the nsel admissions), then -1
   __syncthreads();
   int32_t* out = P.indices + out_off + u.unit * B;
+  // (with the compact cache: position and staged row by rank, where the first-digit
+  // histogram was)
+  int32_t* rpos = reinterpret_cast<int32_t*>(hist0);
+  int32_t* rslot = rpos + kMaxPoolCand;   // ranks < nsel <= C <= kMaxPoolCand
   for (int e = tid; e < nsel; e += NT) {
     const int pos = adm[e];
     int rank = 0;
     for (int f = 0; f < nsel; ++f) rank += (adm[f] < pos);
     out[rank] = pos;
+    if (P.k_out) {
+      rpos[rank] = pos;
+      rslot[rank] = adm_slot[e];
+    }
   }
   for (int r = nsel + tid; r < B; r += NT) out[r] = -1;
   if (order)
     for (int r = nsel + tid; r < B; r += NT) order[r] = -1;
   if (margins)
     for (int r = nsel + tid; r < B; r += NT) margins[r] = 0.f;
+  if (P.k_out) {
+    __syncthreads();
+    write_compact_cache<NT>(P, u, Lc, nsel, nsel, rpos, rslot, krow);
+  }
 }
 
 template <int NT>
@@ -751,6 +816,7 @@ static_assert(kRowChunks * 256 * sizeof(uint4) >= kBins * sizeof(uint32_t), "his
 static_assert(kRowChunks * 256 * sizeof(uint4) >= 2 * (256 * kPoolRun * kPoolRuns + 256) * sizeof(float),
               "pool tiles fit");
 static_assert(kRowChunks * 256 * sizeof(uint4) >= kTieCap * sizeof(int32_t), "tie list fits");
+static_assert(2 * kMaxPoolCand <= kBins, "ranked positions and rows fit the first-digit histogram's place");
 // both parameter blocks of a multi-profile launch fit the 32764-byte kernel
 // parameter space
 static_assert(sizeof(SelectParams) + sizeof(ProfileTable) + 64 <= 32764, "profile table fits");

@@ -22,7 +22,7 @@ EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evi
            "kv_evict_plan_set_debug", "kv_evict_plan_set_kv_strides",
            "kv_evict_score", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
            "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
-           "kv_evict_select_profiles_workspace", "kv_evict_gather",
+           "kv_evict_select_profiles_workspace", "kv_evict_gather", "kv_evict_select_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
 
 
@@ -70,6 +70,7 @@ def _lib():
         lib.kv_evict_select_profiles.argtypes = [vp, i32] + [vp] * 10
         lib.kv_evict_select_profiles_workspace.argtypes = [vp, i32, vp]
         lib.kv_evict_gather.argtypes = [vp] * 7
+        lib.kv_evict_select_gather.argtypes = [vp] * 14
         lib.kv_evict_status.argtypes = [vp, vp, vp]
         lib.kv_evict_profile.argtypes = [i32, vp, i32, vp, vp]
         lib.kv_evict_strerror.argtypes = [ctypes.c_int]
@@ -266,6 +267,22 @@ class Plan:
         _check(_lib().kv_evict_gather(self._h, _ptr(k), _ptr(v), _ptr(indices), _ptr(k_out),
                                       _ptr(v_out), _stream_ptr(stream)), "kv_evict_gather")
 
+    def select_gather(self, mu, sigma, k, v, lambda1, lambda2, indices, k_out, v_out, ws, order=None,
+                      margins=None, stream=None):
+        """kv_evict_select_gather: select, then the compact cache, in one launch (the
+        outputs of select followed by gather). v (and k) may be pinned CPU tensors."""
+        for name, t in (("k", k), ("v", v)):
+            dev = getattr(t, "device", None)
+            if dev is not None and getattr(dev, "type", None) == "cpu" and not t.is_pinned():
+                raise ValueError(f"select_gather: {name} is a pageable CPU tensor; pin it or move it to the GPU")
+        l1 = np.ascontiguousarray(lambda1, dtype=np.float32)
+        l2 = np.ascontiguousarray(lambda2, dtype=np.float32)
+        assert l1.shape == (self.spec["num_layers"],) and l2.shape == l1.shape
+        _check(_lib().kv_evict_select_gather(self._h, _ptr(mu), _ptr(sigma), _ptr(k), _ptr(v),
+                                             l1.ctypes.data, l2.ctypes.data, _ptr(indices), _ptr(order),
+                                             _ptr(margins), _ptr(k_out), _ptr(v_out), _ptr(ws),
+                                             _stream_ptr(stream)), "kv_evict_select_gather")
+
     def status(self, ws, stream=None) -> int:
         """Synchronise, return the device status (KVE_OK, KVE_ETIMEOUT or KVE_ECUDA) of
         ws and clear it; ws = None reads the error word of select_noalloc."""
@@ -310,9 +327,14 @@ class Buffers:
         self.ws = torch.empty(plan.workspace_bytes, dtype=torch.uint8, device=device)
 
 
-def run_step(plan: Plan, bufs: Buffers, q_win, k, v, lambda1, lambda2, stream=None):
-    """The whole eviction step: score, select, gather (three library calls)."""
+def run_step(plan: Plan, bufs: Buffers, q_win, k, v, lambda1, lambda2, stream=None, fused=True):
+    """The whole eviction step: score, then select with the compact cache in one call
+    (fused), or select and gather as two calls."""
     plan.score(q_win, k, bufs.mu, bufs.sigma, bufs.ws, stream)
+    if fused:
+        plan.select_gather(bufs.mu, bufs.sigma, k, v, lambda1, lambda2, bufs.indices, bufs.k_out,
+                           bufs.v_out, bufs.ws, bufs.order, bufs.margins, stream)
+        return
     plan.select(bufs.mu, bufs.sigma, k, lambda1, lambda2, bufs.indices, bufs.ws, bufs.order,
                 bufs.margins, stream)
     plan.gather(k, v, bufs.indices, bufs.k_out, bufs.v_out, stream)
