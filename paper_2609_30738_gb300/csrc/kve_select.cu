@@ -23,6 +23,7 @@
 #include <mutex>
 
 #include "kve_internal.h"
+#include "kve_ptx.cuh"
 
 namespace kve {
 namespace {
@@ -226,6 +227,10 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
   for (int b = tid; b < kBins; b += NT) hist0[b] = 0;
   __syncthreads();
   // 1. pooled base score as ordered keys (and the histogram of their top 12 bits)
+  // L2 policies of the pooling: the keys are read back by the scan below (evict last),
+  // mu and sigma are read once here (evict first)
+  const uint64_t kpol = l2_policy_evict_last();
+  const uint64_t fpol = l2_policy_evict_first();
   if (h == 3) {
     // kernel 7 (the default): groups of 4 consecutive outputs that are 16-byte
     // aligned in mu, sigma and keys, each from three 16-byte loads per array (inputs
@@ -240,7 +245,11 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
         const float4* s4 = reinterpret_cast<const float4*>(sg + i - 4);
 #pragma unroll
         for (int c = 0; c < 3; ++c) {
-          const float4 am = __ldg(m4 + c), as = __ldg(s4 + c);
+          float4 am, as;
+          asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                       : "=f"(am.x), "=f"(am.y), "=f"(am.z), "=f"(am.w) : "l"(m4 + c), "l"(fpol));
+          asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                       : "=f"(as.x), "=f"(as.y), "=f"(as.z), "=f"(as.w) : "l"(s4 + c), "l"(fpol));
           xm[4 * c] = am.x;
           xm[4 * c + 1] = am.y;
           xm[4 * c + 2] = am.z;
@@ -278,7 +287,8 @@ __global__ void __launch_bounds__(NT, NT <= 256 ? 2 : 1) select_kernel(const __g
 #pragma unroll
       for (int r = 0; r < 4; ++r) kk[r] = ord_key(fmaf(lambda1, os[r], om[r]));
       if (i >= 0 && i + 4 <= Lc) {
-        *reinterpret_cast<uint4*>(keys + i) = make_uint4(kk[0], kk[1], kk[2], kk[3]);
+        asm volatile("st.global.L2::cache_hint.v4.u32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(keys + i), "r"(kk[0]),
+                     "r"(kk[1]), "r"(kk[2]), "r"(kk[3]), "l"(kpol) : "memory");
         // consecutive outputs often share the top digit: one atomic per run
         uint32_t bin = kk[0] >> 20, cnt = 1;
 #pragma unroll
