@@ -158,6 +158,20 @@ kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win,
                           const uint16_t* k, float* mu, float* sigma, void* ws,
                           void* stream);
 
+/* Steps 1-2 as kv_evict_score when the softmax normaliser of every window row is
+ * already known -- a prefill attention kernel computes it for its own output (Section
+ * 3.2 scores with the prefill's existing attention). lse [N_L][n_req][Hq][W] fp32 in
+ * q_win's row order (device memory) holds, for the row at position L_r - W + w,
+ *   lse = ln sum_{i <= L_r - W + w} exp(q . k_i / sqrt(d))   (natural log),
+ * so that A[r][i] = exp(q . k_i / sqrt(d) - lse). The library then needs only the
+ * column pass of Eq. 1 and Eq. 3 over the prefix: one pass of the score kernel
+ * instead of two. mu and sigma are exactly as accurate as lse is; a row's lse that is
+ * not finite makes its terms undefined. Reads q_win, k and lse; writes mu and sigma;
+ * uses ws as scratch. */
+kve_status kv_evict_score_lse(const kve_plan* plan, const uint16_t* q_win,
+                              const uint16_t* k, const float* lse, float* mu,
+                              float* sigma, void* ws, void* stream);
+
 /* Steps 1-2 as kv_evict_score, together with the window rows' own attention output.
  * Section 3.2 scores the tokens with the prefill's existing attention; the window rows'
  * attention (the last W positions of every query head) is computed here anyway, so in

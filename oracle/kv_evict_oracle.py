@@ -11,6 +11,8 @@ float64 from the bf16-decoded inputs, in the paper's order:
 
   window_attention   Section 3.1, context of Eq. 1: softmax attention A[q, i] of
                      the window queries over the causal prefix.
+  window_lse         the same rows' natural-log softmax normalisers (what a prefill's
+                     attention computes for its own output; input of the one-pass score).
   mean_attention     Eq. 1: mu_i = (1/|W|) sum_q A[q, i].
   dispersion         Eq. 3: sample standard deviation, divisor |W| - 1.
   max_pool           Section 3.1: the baselines' max-pooling of the scores.
@@ -84,6 +86,20 @@ def window_attention(q: np.ndarray, k: np.ndarray, L: int, W: int, G: int) -> np
     row_max = logits.max(axis=1, keepdims=True)
     e = np.where(visible, np.exp(logits - row_max), 0.0)
     return e / e.sum(axis=1, keepdims=True)
+
+
+def window_lse(q: np.ndarray, k: np.ndarray, L: int, W: int, G: int) -> np.ndarray:
+    """The natural-log softmax normaliser of every window row: ln sum_i exp(q_r . k_i /
+    sqrt(d)) over the keys the row sees (the same causal mask as window_attention), so
+    that A[r, i] = exp(q_r . k_i / sqrt(d) - lse_r) on those keys."""
+    n, d = q.shape
+    assert k.shape == (L, d) and n == G * W
+    logits = (q @ k.T) / math.sqrt(d)
+    pos = window_positions(L, W, G)
+    visible = np.arange(L)[None, :] <= pos[:, None]
+    logits = np.where(visible, logits, -np.inf)
+    row_max = logits.max(axis=1)
+    return row_max + np.log(np.where(visible, np.exp(logits - row_max[:, None]), 0.0).sum(axis=1))
 
 
 def mean_attention(A: np.ndarray) -> np.ndarray:

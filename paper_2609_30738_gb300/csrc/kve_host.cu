@@ -269,8 +269,10 @@ namespace {
 
 // The score step, with the window output when v is given (o_win, attn_ws then too).
 kve_status score_impl(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, const uint16_t* v,
-                      float* mu, float* sigma, uint16_t* o_win, void* ws, void* attn_ws, void* stream) {
+                      float* mu, float* sigma, uint16_t* o_win, void* ws, void* attn_ws, void* stream,
+                      const float* lse = nullptr) {
   if (!plan || !q_win || !k || !mu || !sigma || !ws) return KVE_EINVAL;
+  if (lse && (v || !aligned(lse, 4))) return KVE_EINVAL;
   if (!aligned(q_win, 128) || !aligned(k, 128) || !aligned(mu, 16) || !aligned(sigma, 16) || !aligned(ws, 256))
     return KVE_EINVAL;
   if (v && (!o_win || !attn_ws || !aligned(v, 128) || !aligned(o_win, 16) || !aligned(attn_ws, 256)))
@@ -298,6 +300,7 @@ kve_status score_impl(const kve_plan* plan, const uint16_t* q_win, const uint16_
   p.partial = reinterpret_cast<float2*>(w + plan->ws.partial);
   p.beta = reinterpret_cast<unsigned long long*>(w + plan->ws.beta);
   p.o_part = static_cast<float*>(attn_ws);
+  p.lse = lse;
   const int64_t ctas = std::min<int64_t>(sms, g.n_items);
   p.lag = score_lag(g, ctas);
   if (kve::launch_score(*plan, tm_q, tm_k, v ? &tm_v : nullptr, p, static_cast<int>(ctas), st) != cudaSuccess)
@@ -313,6 +316,12 @@ extern "C" {
 kve_status kv_evict_score(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, float* mu,
                           float* sigma, void* ws, void* stream) {
   return score_impl(plan, q_win, k, nullptr, mu, sigma, nullptr, ws, nullptr, stream);
+}
+
+kve_status kv_evict_score_lse(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k, const float* lse,
+                              float* mu, float* sigma, void* ws, void* stream) {
+  if (!lse) return KVE_EINVAL;
+  return score_impl(plan, q_win, k, nullptr, mu, sigma, nullptr, ws, nullptr, stream, lse);
 }
 
 kve_status kv_evict_score_attn(const kve_plan* plan, const uint16_t* q_win, const uint16_t* k,

@@ -132,6 +132,8 @@ struct ScoreParams {
   float2* partial;
   unsigned long long* beta;   // low word: beta bits, high word: 1 once written
   float* o_part;              // window output: fp32 [n_items][kMaxRows][d] per column item
+  const float* lse;           // given normalisers: natural-log softmax normaliser of every window
+                              // row in q_win's row order (the column pass only), or null
 };
 
 struct SelectParams {

@@ -641,6 +641,22 @@ __device__ __forceinline__ bool try_stage_beta(const ScoreParams& P, ScoreCtl& c
   return stage_beta(P, ctl, w, slot);
 }
 
+// Phase-1 item with given normalisers (P.lse, natural log): stage -beta = -log2(e) * lse
+// of the unit's rows; nothing to wait for.
+__device__ __forceinline__ void stage_lse(const ScoreParams& P, ScoreCtl& ctl, int64_t unit, uint32_t slot) {
+  constexpr float kLog2e = 1.4426950408889634f;
+  const UnitInfo u = unit_info(P.g, unit);
+  const float* l = P.lse + u.q_row0;
+  const int n = P.g.n_rows;
+  const int r0 = 4 * (threadIdx.x & 31);
+  float4 b;
+  b.x = r0 + 0 < n ? fmaf(-kLog2e, l[r0 + 0], kColScale) : -INFINITY;
+  b.y = r0 + 1 < n ? fmaf(-kLog2e, l[r0 + 1], kColScale) : -INFINITY;
+  b.z = r0 + 2 < n ? fmaf(-kLog2e, l[r0 + 2], kColScale) : -INFINITY;
+  b.w = r0 + 3 < n ? fmaf(-kLog2e, l[r0 + 3], kColScale) : -INFINITY;
+  reinterpret_cast<float4*>(ctl.nbeta[slot])[threadIdx.x & 31] = b;
+}
+
 // Phase-1 item: wait (bounded) for the unit's merged statistics and stage -beta.
 __device__ __forceinline__ bool sync_colstats(const ScoreParams& P, ScoreCtl& ctl, int64_t unit,
                                               uint32_t slot) {
@@ -748,7 +764,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool have = true;
         if (ctl.abort) {
           have = false;
-        } else if (jr < own && jr - jc <= P.lag) {
+        } else if (!P.lse && jr < own && jr - jc <= P.lag) {
+          // (with given normalisers there are no phase-0 items)
           cl.phase = 0;
           cl.p = blockIdx.x + jr * G;
           ++jr;
@@ -1071,7 +1088,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = post_merge(job);
         }
       } else {
-        ok = sync_colstats(P, ctl, d.unit, slot);
+        if (P.lse)
+          stage_lse(P, ctl, d.unit, slot);
+        else
+          ok = sync_colstats(P, ctl, d.unit, slot);
         __syncwarp();
         if (lane == 0) {
           mbar_arrive(&ctl.beta_full[slot]);

@@ -20,7 +20,7 @@ KVE_OK, KVE_EINVAL, KVE_ECUDA, KVE_ETIMEOUT, KVE_ENOMEM = range(5)
 # Names declared in include/kv_evict.h.
 EXPORTS = ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_destroy",
            "kv_evict_plan_set_debug", "kv_evict_plan_set_kv_strides",
-           "kv_evict_score", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
+           "kv_evict_score", "kv_evict_score_lse", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
            "kv_evict_select", "kv_evict_select_noalloc", "kv_evict_select_profiles",
            "kv_evict_select_profiles_workspace", "kv_evict_gather", "kv_evict_select_gather",
            "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid", "kv_evict_strerror")
@@ -63,6 +63,7 @@ def _lib():
         lib.kv_evict_plan_set_debug.argtypes = [vp, ctypes.c_uint64, i32]
         lib.kv_evict_plan_set_kv_strides.argtypes = [vp, vp, vp]
         lib.kv_evict_score.argtypes = [vp] * 7
+        lib.kv_evict_score_lse.argtypes = [vp] * 8
         lib.kv_evict_score_attn.argtypes = [vp] * 10
         lib.kv_evict_score_attn_workspace.argtypes = [vp, vp]
         lib.kv_evict_select.argtypes = [vp] * 11
@@ -77,10 +78,11 @@ def _lib():
         lib.kv_evict_strerror.restype = ctypes.c_char_p
         for name in ("kv_evict_plan", "kv_evict_plan_layered", "kv_evict_plan_ex", "kv_evict_plan_set_debug",
                      "kv_evict_plan_set_kv_strides",
-                     "kv_evict_score", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
+                     "kv_evict_score", "kv_evict_score_lse", "kv_evict_score_attn", "kv_evict_score_attn_workspace",
                      "kv_evict_select", "kv_evict_select_noalloc",
                      "kv_evict_select_profiles", "kv_evict_select_profiles_workspace", "kv_evict_gather",
-                     "kv_evict_status", "kv_evict_profile", "kv_evict_budget_pyramid"):
+                     "kv_evict_select_gather", "kv_evict_status", "kv_evict_profile",
+                     "kv_evict_budget_pyramid"):
             getattr(lib, name).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -196,6 +198,12 @@ class Plan:
     def score(self, q_win, k, mu, sigma, ws, stream=None):
         _check(_lib().kv_evict_score(self._h, _ptr(q_win), _ptr(k), _ptr(mu), _ptr(sigma), _ptr(ws),
                                      _stream_ptr(stream)), "kv_evict_score")
+
+    def score_lse(self, q_win, k, lse, mu, sigma, ws, stream=None):
+        """kv_evict_score_lse: the column pass only, given every window row's natural-log
+        softmax normaliser lse (fp32, q_win's row order)."""
+        _check(_lib().kv_evict_score_lse(self._h, _ptr(q_win), _ptr(k), _ptr(lse), _ptr(mu), _ptr(sigma),
+                                         _ptr(ws), _stream_ptr(stream)), "kv_evict_score_lse")
 
     def score_attn_workspace(self) -> int:
         """Bytes of the second scratch buffer of score_attn."""

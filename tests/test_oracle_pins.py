@@ -96,6 +96,32 @@ def test_uniform_keys_closed_form():
     assert abs(mu[0] - np.mean([1.0 / (L - W + w + 1) for w in range(W)])) < 1e-15
 
 
+def test_window_lse_closed_form_and_library():
+    """The window rows' normaliser: equal keys give c_r + ln(p_r + 1) (closed form); random
+    rows equal scipy's logsumexp over each row's visible prefix; exp(l - lse) over the
+    visible keys sums to 1 and equals window_attention's row."""
+    rng = np.random.default_rng(41)
+    L, W, G, d = 20, 4, 3, 8
+    kv = rng.standard_normal(d)
+    k = np.tile(kv, (L, 1))
+    q = rng.standard_normal((G * W, d)) * 3.0
+    lse = O.window_lse(q, k, L, W, G)
+    for r in range(G * W):
+        p = L - W + (r % W)
+        c = float(np.dot(q[r], kv)) / math.sqrt(d)
+        assert abs(lse[r] - (c + math.log(p + 1))) < 1e-12
+    L, W, G, d = 33, 6, 2, 16
+    q, k = _rand_unit(rng, L, W, G, d, scale=4.0)
+    lse = O.window_lse(q, k, L, W, G)
+    A = O.window_attention(q, k, L, W, G)
+    for r in range(G * W):
+        p = L - W + (r % W)
+        logits = np.array([np.dot(q[r], k[i]) for i in range(p + 1)]) / math.sqrt(d)
+        assert abs(lse[r] - scipy.special.logsumexp(logits)) < 1e-12
+        np.testing.assert_allclose(np.exp(logits - lse[r]), A[r, :p + 1], rtol=1e-12, atol=1e-300)
+        assert abs(np.exp(logits - lse[r]).sum() - 1.0) < 1e-12
+
+
 def test_identical_rows_give_zero_sigma():
     """W = 1 and G identical query heads: every row is the same distribution."""
     rng = np.random.default_rng(5)
