@@ -47,8 +47,8 @@ FALLBACK_HBM_GBS = 6800.0
 # from the ncu capture summarised in profiles/, valid only for the sources it was taken
 # on (sha256 over csrc/kve_score.cu and csrc/kve_host.cu, which sets the schedule); per
 # launch of the full workload.
-SCORE_TRAFFIC = {"source_sha256": "536cc3f2475aa8a40d4a1adab4a27ac997f7eb9b03b4eebd3cc0d4d7a6c6efcc",
-                 "bytes_per_launch": 2173897728 + 74817024}
+SCORE_TRAFFIC = {"source_sha256": "60b3a57416c0a61c7b7c3b1774a219755c992425eaef2ae96c39b9cac38a0974",
+                 "bytes_per_launch": 2172808960 + 74820352}
 
 
 def _score_source_sha():
