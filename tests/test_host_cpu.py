@@ -246,6 +246,36 @@ def test_noalloc_size_limit_counts_units_per_layer_without_gpu():
                                        fake, None, None, None) == K.KVE_EINVAL
 
 
+def test_fused_and_given_normaliser_calls_validate_without_gpu():
+    """kv_evict_select_gather and kv_evict_score_lse refuse null and misaligned
+    arguments, and the binding refuses a pageable value tensor, before any launch."""
+    _need_lib()
+    torch = pytest.importorskip("torch")
+    from paper_2609_30738_gb300 import kv_evict as K
+    lib = K.library()
+    p = K.Plan(_spec(num_layers=1), [300])
+    assert lib.kv_evict_score_lse(p._h, None, None, None, None, None, None, None) == K.KVE_EINVAL
+    good, odd = ctypes.c_void_p(1 << 20), ctypes.c_void_p((1 << 20) + 2)
+    # lse must be 4-byte aligned; the check comes before any CUDA call
+    assert lib.kv_evict_score_lse(p._h, good, good, odd, good, good, good, None) == K.KVE_EINVAL
+    lam = np.zeros(1, np.float32)
+    assert lib.kv_evict_select_gather(None, good, good, good, good, lam.ctypes.data, lam.ctypes.data, good,
+                                      None, None, good, good, good, None) == K.KVE_EINVAL
+    assert lib.kv_evict_select_gather(p._h, good, good, good, None, lam.ctypes.data, lam.ctypes.data, good,
+                                      None, None, good, good, good, None) == K.KVE_EINVAL
+    # misaligned mu, then a misaligned output row block
+    assert lib.kv_evict_select_gather(p._h, odd, good, good, good, lam.ctypes.data, lam.ctypes.data, good,
+                                      None, None, good, good, good, None) == K.KVE_EINVAL
+    assert lib.kv_evict_select_gather(p._h, good, good, good, good, lam.ctypes.data, lam.ctypes.data, good,
+                                      None, None, odd, good, good, None) == K.KVE_EINVAL
+    k = torch.zeros((1, 8, 300, 128), dtype=torch.bfloat16)   # pageable
+    mu = torch.zeros(8 * 300, dtype=torch.float32)
+    idx = torch.zeros((8, 64), dtype=torch.int32)
+    out = torch.zeros((8, 96, 128), dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        p.select_gather(mu, mu, k, k, lam, lam, idx, out, out, mu)
+
+
 def test_kv_strides_validation_without_gpu():
     """kv_evict_plan_set_kv_strides: strides in elements (layer, KV head, token), each a
     multiple of 8 and below 2^37, the token stride at least d; NULL restores the dense
