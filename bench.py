@@ -1,8 +1,11 @@
 """Benchmark of the end-of-prefill diversified KV-eviction step on GB300.
 
 One step = the whole path for one call of a Mistral-7B-shaped workload: score
-(window attention, mu, sigma), select (pooling, top-4B, greedy MMR) and gather
-(compact K/V cache). The default workload is "mistral-32layer-L32768-B64": one
+(window attention, mu, sigma), then select (pooling, top-4B, greedy MMR) with the
+gather (compact K/V cache) in the same launch. Beside the step the line reports the
+window-output pass, the one-pass score given the window rows' normalisers, the end-to-
+end call from host buffers and the oracle's throughput. The default workload is
+"mistral-32layer-L32768-B64": one
 request of 32 layers x 8 KV heads (256 units), prefix 32768, window 32, budget 64,
 lambda = (0.5, -0.5). --workload names any of the full-size workloads.
 
